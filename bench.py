@@ -1,0 +1,441 @@
+#!/usr/bin/env python
+"""Benchmark of the Seed-Q decode-fused GEMV on GB300.
+
+A step is one pass of the hot path over every tensor of the workload at batch
+n: the decoder plan is resident, each tensor's compressed stream is in HBM, and
+y = W_hat x is computed for all tensors back to back on one stream.  Default
+workload: the Llama-2-7B-shaped layer set (q, k, v, o 4096x4096; gate, up
+11008x4096; down 4096x11008) at 4.0 bits/weight, batch 1.
+
+Prints one JSON line (rank 0).  --impl reference times the CPU oracle instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "decode tokens/s & effective weight GB/s at batch 1; % of roofline"
+FLUSH_BYTES = 512 << 20  # > 129 MB L2: written between timed steps
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--workload", default="c1")
+    p.add_argument("--batch", type=int, default=1)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    return p.parse_args()
+
+
+def load_schedule(name):
+    from paper_2609_38477_gb300 import workloads as W
+
+    d = json.load(open(os.path.join(ROOT, "tests", "golden", f"schedule_{name}.json")))
+    if d["a_rho_checksum"] != W.a_rho_checksum(W.WORKLOADS[name]):
+        raise RuntimeError(f"importance inputs of {name} differ from the stored schedule's")
+    return d
+
+
+def measured_peaks():
+    try:
+        return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except Exception:
+        return None
+
+
+# ------------------------------------------------------------------ clocks
+
+class Clocks:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: str):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", self.index, f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if not self.proc:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 8:
+                continue
+            try:
+                sm.append(float(f[0]))
+                mx.append(float(f[1]))
+            except ValueError:
+                continue
+            for nme, v in zip(names, f[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(nme)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+def gpu_index(local_rank: int) -> str:
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    if vis:
+        return vis.split(",")[local_rank].strip()
+    return str(local_rank)
+
+
+# ------------------------------------------------------------- distributed
+
+def dist_init():
+    import torch
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    return rank, world, local
+
+
+def dist_max(v: float) -> float:
+    import torch
+    import torch.distributed as dist
+
+    if not (dist.is_available() and dist.is_initialized()):
+        return v
+    dev = "cuda" if torch.cuda.is_available() and dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([v], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def dist_barrier():
+    import torch.distributed as dist
+
+    if dist.is_available() and dist.is_initialized():
+        dist.barrier()
+
+
+# ------------------------------------------------------------ algorithmic
+
+def algorithmic_counts(w, gts, sched, n):
+    """Per-step algorithmic work: warp-instructions of the issue model
+    (per weight: k_b LFSR states, k_b integer MACs, one convert, n FMAs) and
+    HBM bytes (payload, plan rows read, x, y)."""
+    import numpy as np
+
+    rungs = sched["rungs"]
+    J = len(rungs)
+    warp_inst, bytes_, ksum, blocks = 0.0, 0, 0, 0
+    for gt in gts:
+        t = gt.spec
+        rm = gt.layer.rung_map()
+        cnt = np.bincount(rm.ravel(), minlength=J)
+        for j, (S, k) in enumerate(rungs):
+            warp_inst += cnt[j] * 8 * (2 * k + 1 + n) / 32.0
+            ksum += int(cnt[j]) * k
+        blocks += int(cnt.sum())
+        bytes_ += (gt.bits + 7) // 8 + t.R * (8 + 4 * (J - 1)) + 2 * n * t.C + 4 * n * t.R
+    return warp_inst, bytes_, ksum / blocks
+
+
+def traffic_per_launch(kernel_hash: str):
+    path = os.path.join(ROOT, "profiles", "k_gemv_c1_dram_traffic.txt")
+    if not os.path.exists(path):
+        return None
+    kv = {}
+    for line in open(path):
+        if "=" in line and not line.startswith("#"):
+            k, v = line.strip().split("=", 1)
+            kv[k.strip()] = v.strip()
+    if kv.get("kernel_source_sha256") != kernel_hash:
+        return None
+    try:
+        return float(kv["dram_bytes_per_launch"])
+    except (KeyError, ValueError):
+        return None
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for f in ("gemv.cu", "seedq_internal.cuh"):
+        h.update(open(os.path.join(ROOT, "paper_2609_38477_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+# ------------------------------------------------------------- CPU oracle
+
+def oracle_sample(w, sched, n, target_s: float, nthreads: int):
+    """Prepare a bounded sample of the workload for the oracle: the first rows
+    of every tensor, as many as ~target_s seconds of oracle work allow.
+    Returns (run, fraction, description)."""
+    sys.path.insert(0, os.path.join(ROOT, "oracle"))
+    import oracle as O
+    from paper_2609_38477_gb300 import workloads as W
+
+    s = O.Sched([tuple(r) for r in sched["rungs"]], sched["theta"], sched["j_tie"], sched["q"])
+    ts = [O.Tensor(t.R, t.C, *W.importance(w, i)) for i, t in enumerate(w.tensors)]
+    xs = [W.x_bf16(w, i, n) for i in range(len(w.tensors))]
+    # Calibrate on 32 rows of the first tensor.
+    t0 = ts[0]
+    st, bits = t0.synth_pack_rows(s, sched["tie_count"][0], W.payload_key(w, 0), 0, 32,
+                                  32 * t0.C * 6)
+    c0 = time.perf_counter()
+    t0.decode_gemv_threads(s, sched["tie_count"][0], st, bits, xs[0], nthreads, 0, 32)
+    rate = 32 * t0.C / max(time.perf_counter() - c0, 1e-6)  # weights / s
+    frac = min(1.0, target_s * rate / w.weights)
+    jobs = []
+    for i, (t, ot) in enumerate(zip(w.tensors, ts)):
+        rows = max(1, int(round(frac * t.R)))
+        st, bits = ot.synth_pack_rows(s, sched["tie_count"][i], W.payload_key(w, i), 0, rows,
+                                      rows * t.C * 6)
+        jobs.append((ot, sched["tie_count"][i], st, bits, xs[i], rows))
+    sample_w = sum(rows * t.C for (ot, _, _, _, _, rows), t in zip(jobs, w.tensors))
+    frac = sample_w / w.weights
+
+    def run():
+        used = 0
+        for ot, T, st, bits, x, rows in jobs:
+            _, used = ot.decode_gemv_threads(s, T, st, bits, x, nthreads, 0, rows)
+        return used
+
+    desc = (f"oracle decode (Alg. 2) + fp64 GEMV of the first {frac * 100:.1f}% of rows of every "
+            f"tensor ({sample_w / 1e6:.1f} M of {w.weights / 1e6:.1f} M weights), batch {n}; "
+            f"tokens/s extrapolated to the full workload")
+    return run, frac, desc
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def reference_arm(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    from paper_2609_38477_gb300 import workloads as W
+
+    w = W.WORKLOADS[args.workload]
+    sched = load_schedule(args.workload)
+    n = args.batch
+    cores = cpu_cores()
+    total_steps = args.steps + args.warmup
+    per_step = max(0.5, min(6.0, 150.0 / max(total_steps, 1)))
+    run, frac, desc = oracle_sample(w, sched, n, per_step, cores)
+    for _ in range(args.warmup):
+        run()
+    times, used = [], cores
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        used = run()
+        times.append(time.perf_counter() - t0)
+    step = statistics.mean(times) / frac  # full-workload seconds per step
+    value = n / step
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": step * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": f"{w.name}: {w.description}", "batch": n},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": used, "kind": "oracle",
+                         "sample": desc},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------- our arm
+
+def our_arm(args):
+    import numpy as np
+    import torch
+
+    rank, world, local = dist_init()
+    torch.cuda.set_device(local)
+    import __graft_entry__ as GE
+
+    GE.build()
+    from paper_2609_38477_gb300 import workload_gpu as G
+    from paper_2609_38477_gb300 import workloads as W
+
+    w = W.WORKLOADS[args.workload]
+    sched = load_schedule(args.workload)
+    n = args.batch
+    gts = G.prepare_workload(w, sched, max_batch=n)
+    xs = [G.x_device(w, i, n) for i in range(len(w.tensors))]
+    ys = [torch.empty((n, t.R), dtype=torch.float32, device="cuda") for t in w.tensors]
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.current_stream()
+    h = stream.cuda_stream
+
+    def step():
+        for gt, x, y in zip(gts, xs, ys):
+            if n == 1:
+                gt.layer.gemv(x, y, h)
+            else:
+                gt.layer.gemm_small_batch(x, n, y, h)
+
+    for _ in range(max(args.warmup, 3)):
+        flush.zero_()
+        step()
+    torch.cuda.synchronize()
+
+    # Timed steps: device time of each step (CUDA events on the launching stream).
+    clocks = Clocks(gpu_index(local))
+    dist_barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    for a, b in ev:
+        flush.zero_()
+        a.record(stream)
+        step()
+        b.record(stream)
+    torch.cuda.synchronize()
+    dist_barrier()
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    # Per-call timing of the fused kernel (same launches, events between calls).
+    per_call = [[] for _ in gts]
+    for _ in range(args.steps):
+        flush.zero_()
+        evs = [torch.cuda.Event(enable_timing=True) for _ in range(len(gts) + 1)]
+        evs[0].record(stream)
+        for i, (gt, x, y) in enumerate(zip(gts, xs, ys)):
+            if n == 1:
+                gt.layer.gemv(x, y, h)
+            else:
+                gt.layer.gemm_small_batch(x, n, y, h)
+            evs[i + 1].record(stream)
+        torch.cuda.synchronize()
+        for i in range(len(gts)):
+            per_call[i].append(evs[i].elapsed_time(evs[i + 1]))
+    clk = clocks.stop()
+
+    # End to end through the C ABI with host buffers: H2D of x, D2H of y.
+    xh = [x.cpu().pin_memory() for x in xs]
+    yh = [torch.empty(y.shape, dtype=torch.float32).pin_memory() for y in ys]
+    h2d = sum(x.numel() * 2 for x in xs)
+    d2h = sum(y.numel() * 4 for y in ys)
+    e2e_ms = []
+    for _ in range(args.steps):
+        flush.zero_()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for xd, xhh in zip(xs, xh):
+            xd.copy_(xhh, non_blocking=True)
+        step()
+        for yd, yhh in zip(ys, yh):
+            yhh.copy_(yd, non_blocking=True)
+        b.record(stream)
+        b.synchronize()
+        e2e_ms.append(a.elapsed_time(b))
+
+    mean_step = dist_max(statistics.mean(step_ms))
+    mean_e2e = dist_max(statistics.mean(e2e_ms))
+    warp_inst, alg_bytes, mean_k = algorithmic_counts(w, gts, sched, n)
+    call_ms = [statistics.mean(v) for v in per_call]
+    kern_ms = sum(call_ms)
+    props = torch.cuda.get_device_properties(local)
+    sms = props.multi_processor_count
+    peaks = measured_peaks()
+    sm_max = (peaks or {}).get("sm_max_mhz") or (clk or {}).get("sm_max_mhz") or 2070.0
+    issue_peak = 4 * sms * sm_max * 1e6 / 1e9  # Gwarp-inst/s
+    hbm_peak = (peaks or {}).get("hbm_gbs") or 6800.0
+    achieved_issue = warp_inst / (kern_ms * 1e-3) / 1e9
+    achieved_hbm = alg_bytes / (kern_ms * 1e-3) / 1e9
+    nbt = 1 if n <= 1 else 2 if n <= 2 else 4 if n <= 4 else 8 if n <= 8 else 16
+    nsplit_tensors = sum(1 for gt in gts if (gt.spec.C // 8) > 1024 // nbt)  # split-K reduce launches
+    stream_bytes = sum((gt.bits + 7) // 8 for gt in gts)
+    value = world * n / (mean_step * 1e-3)
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": mean_step,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "fp32", "data": "synthetic",
+        "config": {
+            "workload": f"{w.name}: {w.description}", "batch": n,
+            "bits_per_weight": sched["mean_bits_per_weight"], "weights": w.weights,
+            "stream_bytes": stream_bytes, "mean_k": round(mean_k, 4),
+            "l2": f"flushed between timed steps ({FLUSH_BYTES >> 20} MiB write)",
+            "parallelism": "replicas" if world > 1 else "single GPU",
+        },
+        "weight_equiv_gbs": 2 * w.weights / (mean_step * 1e-3) / 1e9,
+        "compressed_gbs": stream_bytes / (mean_step * 1e-3) / 1e9,
+        "clocks": clk,
+        "e2e": {"value": world * n / (mean_e2e * 1e-3), "unit": "tokens/s",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": args.steps * (len(gts) + nsplit_tensors),
+        "roofline": {
+            "bound": "alu", "achieved": achieved_issue, "peak": issue_peak,
+            "unit": "Gwarp-inst/s", "frac": achieved_issue / issue_peak,
+            "traffic": traffic_per_launch(kernel_source_hash()),
+            "kernel": "k_gemv (fused decode x GEMV), all tensors of the step",
+            "peak_basis": f"4 warp-inst/clk/SM x {sms} SMs x {sm_max:.0f} MHz",
+            "hbm": {"achieved_gbs": achieved_hbm, "peak_gbs": hbm_peak,
+                    "frac": achieved_hbm / hbm_peak,
+                    "peak_basis": "MEASURED_PEAKS.json hbm_gbs (measured)" if peaks else "fallback"},
+            "per_call_us": {gt.spec.name: round(m * 1e3, 2) for gt, m in zip(gts, call_ms)},
+        },
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cores = cpu_cores()
+        run, frac, desc = oracle_sample(w, sched, n, 10.0, cores)
+        t0 = time.perf_counter()
+        used = run()
+        el = time.perf_counter() - t0
+        line["cpu_baseline"] = {"value": n / (el / frac), "unit": "tokens/s", "cores": used,
+                                "kind": "oracle", "sample": desc}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    for gt in gts:
+        gt.layer.release()
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        reference_arm(args)
+    else:
+        our_arm(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,194 @@
+/*
+ * seedq.h -- C ABI of libseedq.so, a GB300 (sm_103a) implementation of the
+ * inference hot path of Seed-Q ("Security-Enhanced Seed-Based Weight
+ * Quantization for Large Language Models", arxiv 2609.38477): weight blocks
+ * regenerated from LFSR seeds and 4-bit coefficients (Sec. 3.1, Eq. codec)
+ * under the side-information-free rung schedule (Sec. 3.3-3.6, Alg. 2),
+ * consumed straight away by a decode-batch matrix-vector product.
+ *
+ * General rules for every entry point:
+ *  - Pointers marked "device" must point to memory of the current CUDA
+ *    device; pointers marked "host" to ordinary host memory.  The caller owns
+ *    every buffer it passes (stream, x, y, W, outlier values) and the CUDA
+ *    stream.  A seedq_layer owns only the plan derived from its descriptor.
+ *  - `cuda_stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *    stream).  Hot calls (decode, gemv, gemm) only enqueue work on it: they
+ *    allocate nothing, do not synchronize, and return before the work ends.
+ *  - Argument errors are reported synchronously, before any launch, and leave
+ *    nothing enqueued.  SEEDQ_ERR_CUDA means a CUDA call failed; the message
+ *    of the last failure is available from seedq_last_cuda_error_string().
+ *  - A layer may be used from several host threads only if calls on it are
+ *    serialized; different layers are independent.
+ *
+ * Stream format (Sec. 3.1 Eq. rate, Sec. 3.6; the paper leaves the bit order
+ * open and this library fixes it): one little-endian bit string, bit p in
+ * byte p>>3 at bit p&7; a block of rung (S,k) is l = S + 4k + 4 bits, fields
+ * LSB first in the order seed (S bits), shared exponent E (4-bit two's
+ * complement), mantissas t_0..t_{k-1} (4-bit two's complement each); blocks in
+ * row-major order of the column-permuted matrix, no padding between rows.
+ * The LFSR of width S is the window form o_{t+S} = XOR_{i in T_S} o_{t+i}
+ * seeded with the seed's bits (see seedq_lfsr_taps), and entry (i,j) of U(s)
+ * is (x_{ik+j} - 2^{S-1}) / 2^{S-1}, x_n the S-bit window after n clocks.
+ */
+#ifndef SEEDQ_H
+#define SEEDQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  SEEDQ_OK = 0,
+  SEEDQ_ERR_INVALID_ARG = 1,  /* NULL pointer, bad size, non-finite factor */
+  SEEDQ_ERR_STREAM = 2,       /* stream length or buffer size disagrees with the plan */
+  SEEDQ_ERR_SCHEDULE = 3,     /* thresholds not increasing, tie count > tied blocks */
+  SEEDQ_ERR_CUDA = 4,         /* a CUDA runtime call failed */
+  SEEDQ_ERR_NOMEM = 5,        /* device or host allocation failed (prepare only) */
+  SEEDQ_ERR_UNSUPPORTED = 6   /* rung or shape outside what the kernels implement */
+} seedq_status;
+
+/* A rung g = (S, k) of the hull (Sec. 3.1 "We call g = (S,k) a rung").
+ * Supported: S in {8, 10, 12, 14, 16}, k in {2, ..., 6}. */
+typedef struct {
+  int32_t S;
+  int32_t k;
+} seedq_rung;
+
+/* The global decoder table of Sec. 3.6 / Alg. 2 (Require line): hull rungs,
+ * thresholds and floor.  All arrays are host memory, read during prepare only.
+ *   J      number of hull rungs, 1..9, rates strictly increasing.
+ *   theta  J-1 thresholds, strictly increasing: theta[j] = lambda / s_j of
+ *          Eq. ladder, stored as the encoder computed it (the decoder does not
+ *          divide, so encoder and decoder compare the same doubles).
+ *   j_tie  index of the threshold whose tied group is partially demoted
+ *          (App. A.5), or -1.
+ *   q      importance floor of Sec. 3.3 (imp <- max(imp, q)). */
+typedef struct {
+  int32_t J;
+  const seedq_rung *rungs;
+  const double *theta;
+  int32_t j_tie;
+  double q;
+} seedq_schedule;
+
+/* One weight tensor W (R x C) and the per-tensor inputs of Alg. 2.
+ *   rows, cols    R, C; C a multiple of 8, 8 <= C <= 65536; 1 <= R <= 2^24.
+ *   a             host, C floats, finite and >= 0, not all zero: the input
+ *                 second moments (Eq. gamma or Eq. prop).
+ *   rho           host, R floats finite and > 0, or NULL for all ones
+ *                 (output factor of Sec. 3.3 "Output side").
+ *   tie_count     T_t of Alg. 2: the first T_t tied blocks in row-major order
+ *                 take the lower rung.
+ *   n_outliers    0..16 FP16 outlier columns (Sec. 3.5, App. A.6).
+ *   outlier_cols  host, n_outliers distinct column indices in [0, C).
+ *   outlier_vals  device, R x n_outliers binary16 values, row-major; read by
+ *                 every decode/gemv call, so it must outlive the layer.
+ *   max_batch     largest n passed to seedq_gemm_small_batch (1..16); 0 = 16. */
+typedef struct {
+  int64_t rows;
+  int64_t cols;
+  const float *a;
+  const float *rho;
+  int64_t tie_count;
+  int32_t n_outliers;
+  const int32_t *outlier_cols;
+  const uint16_t *outlier_vals;
+  int32_t max_batch;
+} seedq_layer_desc;
+
+typedef struct seedq_layer seedq_layer;
+
+/* Build the decoder plan of one tensor (Alg. 2 lines computing imp, the floor
+ * and the ladder; App. A.7 "Agreement"): column permutation (stable ascending
+ * sort of a), unit-mean block means and row factors in fp64 in a fixed order,
+ * per-row rung breakpoints after the tie pass, per-row bit offsets.  Runs on
+ * the device on `cuda_stream` and waits for it (one-time set-up).  Allocates
+ * the plan's device memory; *out receives the layer.  Errors: INVALID_ARG,
+ * UNSUPPORTED (rung or size), SCHEDULE (theta not increasing, j_tie out of
+ * range, tie_count larger than the tied group), NOMEM, CUDA. */
+seedq_status seedq_layer_prepare(const seedq_layer_desc *desc,
+                                 const seedq_schedule *sched, void *cuda_stream,
+                                 seedq_layer **out);
+
+/* Total payload bits the plan expects for the tensor (sum of l(g_b)). */
+seedq_status seedq_layer_stream_bits(const seedq_layer *layer, uint64_t *bits);
+
+/* Bytes a stream buffer of `bits` payload bits must span: the payload rounded
+ * up to 16 bytes plus a 16-byte guard that the kernels may read (never use). */
+uint64_t seedq_stream_bytes_required(uint64_t bits);
+
+/* Attach the compressed stream (device, caller-owned, 16-byte aligned) to the
+ * layer.  stream_bits must equal seedq_layer_stream_bits and stream_bytes must
+ * be at least seedq_stream_bytes_required(stream_bits); otherwise
+ * SEEDQ_ERR_STREAM.  The buffer must stay valid while the layer is used. */
+seedq_status seedq_layer_bind_stream(seedq_layer *layer, const void *stream,
+                                     uint64_t stream_bits, uint64_t stream_bytes);
+
+/* Free the plan (waits for the device).  NULL is accepted. */
+seedq_status seedq_layer_release(seedq_layer *layer);
+
+/* Alg. 2 in full: every block reconstructed by Eq. codec, written through the
+ * inverse column permutation, outlier columns overwritten (Alg. 2 last lines).
+ * W: device, R x C float32, row-major, original column order.  Values are
+ * exact (each weight is I * 2^(E-S+1) with |I| < 2^21).  Needs a bound stream. */
+seedq_status seedq_decode_weights(const seedq_layer *layer, float *W,
+                                  void *cuda_stream);
+
+/* Rows [row0, row0 + nrows) only; W: device, nrows x C. */
+seedq_status seedq_decode_rows(const seedq_layer *layer, int64_t row0,
+                               int64_t nrows, float *W, void *cuda_stream);
+
+/* y = W_hat x (the matrix-vector product the reconstructed weights feed,
+ * Sec. 1 and App. C; W_hat is never materialized).  x: device, C bfloat16
+ * values (bit patterns) in the original column order; y: device, R float32.
+ * Accumulation in fp32. */
+seedq_status seedq_gemv(const seedq_layer *layer, const uint16_t *x, float *y,
+                        void *cuda_stream);
+
+/* Y = X W_hat^T for n = 1..max_batch activation columns: X device n x C
+ * bfloat16 row-major, Y device n x R float32 row-major (row b of Y is
+ * W_hat x_b).  Each block is reconstructed once and used for all n columns. */
+seedq_status seedq_gemm_small_batch(const seedq_layer *layer, const uint16_t *X,
+                                    int32_t n, float *Y, void *cuda_stream);
+
+/* Host copy of the rung index (0..J-1) of blocks of rows [row0, row0+nrows):
+ * rungs_host receives nrows x (C/8) bytes.  Synchronous. */
+seedq_status seedq_layer_rung_map(const seedq_layer *layer, int64_t row0,
+                                  int64_t nrows, uint8_t *rungs_host);
+
+/* Host copy of the column permutation (C int32): block c of a row holds
+ * original columns perm[8c .. 8c+7].  Synchronous. */
+seedq_status seedq_layer_perm(const seedq_layer *layer, int32_t *perm_host);
+
+/* Host copy of the per-row bit offsets (R+1 uint64, offsets[R] = total). */
+seedq_status seedq_layer_row_offsets(const seedq_layer *layer, uint64_t *offsets_host);
+
+/* Device error flags accumulated by the layer's kernels since prepare (bit 0:
+ * a block offset disagreed with the row offsets; bit 1: unbound stream).
+ * Synchronous; 0 means no fault was seen. */
+seedq_status seedq_last_device_error(const seedq_layer *layer, uint32_t *flags);
+
+/* Tap mask T_S of the width-S LFSR used by the stream format (bit i set when
+ * o_{t+i} feeds o_{t+S}); 0 for widths outside 8..16.  Host function. */
+uint32_t seedq_lfsr_taps(int32_t S);
+
+/* Fill a stream buffer with the synthetic payload of the workload recipe:
+ * block b of the tensor (row-major) draws h = splitmix64 output number b from
+ * state `key` and uses seed = 1 + (h>>32) mod (2^S-1), E = -8 + ((h>>24)&255)
+ * mod 6, t_j = ((h>>4j)&15) - 8 at the rung the plan assigns.  stream: device,
+ * stream_bytes >= seedq_stream_bytes_required(plan bits); zeroed first.  A
+ * benchmark and test input generator, not part of the paper's method. */
+seedq_status seedq_synth_stream(const seedq_layer *layer, uint64_t key,
+                                void *stream, uint64_t stream_bytes,
+                                void *cuda_stream);
+
+const char *seedq_status_string(seedq_status status);
+const char *seedq_last_cuda_error_string(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* SEEDQ_H */

@@ -128,8 +128,9 @@ static void *job_run(void *arg) {
 int or_decode_gemv_threads(const or_factors *f, const or_schedule *s,
                            int64_t tie_count, const uint8_t *stream,
                            uint64_t stream_bits, const uint32_t *taps, int nb,
-                           const uint16_t *x_bf16, double *y, int nthreads) {
-  const int64_t R = f->R, nblk = f->C / 8;
+                           const uint16_t *x_bf16, int64_t r0, int64_t nrows,
+                           double *y, int nthreads) {
+  const int64_t R = r0 + nrows, nblk = f->C / 8;
   if (nthreads < 1) nthreads = 1;
   if (nthreads > 256) nthreads = 256;
   uint8_t *rungs = (uint8_t *)malloc((size_t)(R * nblk));
@@ -149,7 +150,7 @@ int or_decode_gemv_threads(const or_factors *f, const or_schedule *s,
   job_t jobs[256];
   for (int i = 0; i < nthreads; ++i) {
     jobs[i] = (job_t){f, s, stream, taps, rungs, offs, x_bf16, y, nb,
-                      R * i / nthreads, R * (i + 1) / nthreads};
+                      r0 + nrows * i / nthreads, r0 + nrows * (i + 1) / nthreads};
     pthread_create(&th[i], NULL, job_run, &jobs[i]);
   }
   for (int i = 0; i < nthreads; ++i) pthread_join(th[i], NULL);
@@ -212,4 +213,82 @@ void or_synth_rows(const or_factors *f, const or_schedule *s, int64_t tie_count,
       row[outlier_cols[o]] = half_to_float(outlier_vals[r * n_out + o]);
   }
   free(rungs);
+}
+
+/* ---------------- threaded fp64 product straight from synthetic fields ---------------- */
+
+typedef struct {
+  const or_factors *f;
+  const or_schedule *s;
+  int64_t tie_count;
+  uint64_t key;
+  const uint32_t *taps;
+  const uint16_t *x;
+  double *y, *yabs;
+  int nb;
+  int64_t r0, r1;
+} sjob_t;
+
+static void *sjob_run(void *arg) {
+  sjob_t *jb = (sjob_t *)arg;
+  const int64_t C = jb->f->C;
+  float *row = (float *)malloc(sizeof(float) * (size_t)C);
+  for (int64_t r = jb->r0; r < jb->r1; ++r) {
+    or_synth_rows(jb->f, jb->s, jb->tie_count, jb->key, jb->taps, 0, NULL, NULL, r, 1, row);
+    for (int b = 0; b < jb->nb; ++b) {
+      double acc = 0.0, aab = 0.0;
+      for (int64_t c = 0; c < C; ++c) {
+        const double xv = bf16_to_double(jb->x[b * C + c]);
+        acc = acc + (double)row[c] * xv;
+        aab = aab + fabs((double)row[c]) * fabs(xv);
+      }
+      jb->y[b * jb->f->R + r] = acc;
+      if (jb->yabs) jb->yabs[b * jb->f->R + r] = aab;
+    }
+  }
+  free(row);
+  return NULL;
+}
+
+int or_synth_gemv_threads(const or_factors *f, const or_schedule *s, int64_t tie_count,
+                          uint64_t key, const uint32_t *taps, int nb,
+                          const uint16_t *x_bf16, int64_t r0, int64_t nrows, double *y,
+                          double *yabs, int nthreads) {
+  if (nthreads < 1) nthreads = 1;
+  if (nthreads > 256) nthreads = 256;
+  pthread_t th[256];
+  sjob_t jobs[256];
+  for (int i = 0; i < nthreads; ++i) {
+    jobs[i] = (sjob_t){f, s, tie_count, key, taps, x_bf16, y, yabs, nb,
+                       r0 + nrows * i / nthreads, r0 + nrows * (i + 1) / nthreads};
+    pthread_create(&th[i], NULL, sjob_run, &jobs[i]);
+  }
+  for (int i = 0; i < nthreads; ++i) pthread_join(th[i], NULL);
+  return nthreads;
+}
+
+/* Pack rows [r0, r0+nrows) of the synthetic stream into out starting at bit 0
+ * (zeroed by the caller).  Returns the number of bits written. */
+uint64_t or_synth_pack_rows(const or_factors *f, const or_schedule *s, int64_t tie_count,
+                            uint64_t key, int64_t r0, int64_t nrows, uint8_t *out) {
+  const int64_t nb = f->C / 8;
+  uint8_t *rungs = (uint8_t *)malloc((size_t)nb);
+  int64_t remaining = or_tie_remaining(f, s, tie_count, r0);
+  uint64_t pos = 0;
+  for (int64_t r = r0; r < r0 + nrows; ++r) {
+    or_rung_rows_cont(f, s, &remaining, r, 1, rungs);
+    for (int64_t c = 0; c < nb; ++c) {
+      const int S = s->S[rungs[c]], k = s->k[rungs[c]];
+      uint32_t seed;
+      int E, t[6];
+      or_synth_fields(key, (uint64_t)(r * nb + c), S, k, &seed, &E, t);
+      or_write_bits(out, pos, S, seed);
+      or_write_bits(out, pos + (uint64_t)S, 4, (uint64_t)(E & 15));
+      for (int j = 0; j < k; ++j)
+        or_write_bits(out, pos + (uint64_t)(S + 4 + 4 * j), 4, (uint64_t)(t[j] & 15));
+      pos += (uint64_t)or_block_bits(S, k);
+    }
+  }
+  free(rungs);
+  return pos;
 }

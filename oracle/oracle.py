@@ -80,12 +80,16 @@ def lib():
                                          i32p, u16p, C.c_int64, C.c_int64, fp]),
             "or_gemv_f64": (None, [C.c_int64, C.c_int64, fp, C.c_int, u16p, dp]),
             "or_decode_gemv_threads": (C.c_int, [FP, SP, C.c_int64, u8p, C.c_uint64, u32p,
-                                                 C.c_int, u16p, dp, C.c_int]),
+                                                 C.c_int, u16p, C.c_int64, C.c_int64, dp, C.c_int]),
             "or_splitmix64_at": (C.c_uint64, [C.c_uint64, C.c_uint64]),
             "or_synth_fields": (None, [C.c_uint64, C.c_uint64, C.c_int, C.c_int, u32p, ip, ip]),
             "or_synth_pack": (C.c_uint64, [FP, SP, C.c_int64, C.c_uint64, u8p]),
             "or_synth_rows": (None, [FP, SP, C.c_int64, C.c_uint64, u32p, C.c_int, i32p, u16p,
                                      C.c_int64, C.c_int64, fp]),
+            "or_synth_gemv_threads": (C.c_int, [FP, SP, C.c_int64, C.c_uint64, u32p, C.c_int, u16p,
+                                                C.c_int64, C.c_int64, dp, dp, C.c_int]),
+            "or_synth_pack_rows": (C.c_uint64, [FP, SP, C.c_int64, C.c_uint64, C.c_int64,
+                                                C.c_int64, u8p]),
             "or_hull": (C.c_int, [C.c_int, ip, ip, dp, ip]),
             "or_allocate": (C.c_int, [C.c_int, C.POINTER(FP), C.c_int, ip, ip, dp, C.c_double,
                                       C.c_double, dp, ip, dp, i64p, u64p]),
@@ -265,14 +269,36 @@ class Tensor:
                             _p(W, C.c_float))
         return W
 
-    def decode_gemv_threads(self, s, T, stream, stream_bits, x_bf16, nthreads):
+    def synth_gemv(self, s, T, key, x_bf16, r0=0, nrows=None, nthreads=None):
+        """fp64 y = W_hat x and sum |W_hat| |x| for rows [r0, r0+nrows) of the
+        synthetic tensor (nb x nrows arrays)."""
+        nrows = self.R - r0 if nrows is None else nrows
+        x = np.ascontiguousarray(x_bf16, np.uint16)
+        nb = x.size // self.C
+        y = np.zeros((nb, self.R), np.float64)
+        ya = np.zeros((nb, self.R), np.float64)
+        nthreads = nthreads or max(1, min(os.cpu_count() or 1, 64))
+        taps = taps_table()
+        lib().or_synth_gemv_threads(C.byref(self.f), C.byref(s.c), T, key, _p(taps, C.c_uint32), nb,
+                                    _p(x, C.c_uint16), r0, nrows, _p(y, C.c_double),
+                                    _p(ya, C.c_double), nthreads)
+        return y[:, r0:r0 + nrows], ya[:, r0:r0 + nrows]
+
+    def synth_pack_rows(self, s, T, key, r0, nrows, nbits_hint):
+        out = np.zeros((nbits_hint + 7) // 8 + 16, np.uint8)
+        bits = lib().or_synth_pack_rows(C.byref(self.f), C.byref(s.c), T, key, r0, nrows,
+                                        _p(out, C.c_uint8))
+        return out, bits
+
+    def decode_gemv_threads(self, s, T, stream, stream_bits, x_bf16, nthreads, r0=0, nrows=None):
+        nrows = self.R - r0 if nrows is None else nrows
         x = np.ascontiguousarray(x_bf16, np.uint16)
         nb = x.size // self.C
         y = np.zeros((nb, self.R), np.float64)
         taps = taps_table()
         n = lib().or_decode_gemv_threads(C.byref(self.f), C.byref(s.c), T, _p(stream, C.c_uint8),
                                          stream_bits, _p(taps, C.c_uint32), nb,
-                                         _p(x, C.c_uint16), _p(y, C.c_double), nthreads)
+                                         _p(x, C.c_uint16), r0, nrows, _p(y, C.c_double), nthreads)
         if n < 0:
             raise ValueError("stream too short")
         return y, n

@@ -139,13 +139,14 @@ int or_decode_rows(const or_factors *f, const or_schedule *s, int64_t tie_count,
 void or_gemv_f64(int64_t nrows, int64_t C, const float *W, int nb,
                  const uint16_t *x_bf16, double *y);
 
-/* Multi-threaded decode + fp64 GEMV of the whole tensor, used only to time
- * the oracle as a CPU baseline.  Returns the thread count used. */
+/* Multi-threaded decode + fp64 GEMV of rows [r0, r0+nrows) (y is nb x R),
+ * used to time the oracle as a CPU baseline.  Returns the thread count used,
+ * or -1 if the stream is too short. */
 int or_decode_gemv_threads(const or_factors *f, const or_schedule *s,
                            int64_t tie_count, const uint8_t *stream,
                            uint64_t stream_bits, const uint32_t *taps,
-                           int nb, const uint16_t *x_bf16, double *y,
-                           int nthreads);
+                           int nb, const uint16_t *x_bf16, int64_t r0,
+                           int64_t nrows, double *y, int nthreads);
 
 /* ---------------- synthetic payload (counter-based generator) ---------------- */
 
@@ -170,6 +171,19 @@ void or_synth_rows(const or_factors *f, const or_schedule *s, int64_t tie_count,
                    uint64_t key, const uint32_t *taps, int n_out,
                    const int32_t *outlier_cols, const uint16_t *outlier_vals,
                    int64_t r0, int64_t nrows, float *W);
+
+/* y (and, when yabs is not NULL, sum_c |W_rc| |x_c|) for rows [r0, r0+nrows)
+ * of a synthetic tensor, from its fields, in fp64 over nthreads threads.
+ * y and yabs are nb x R (only the requested rows are written). */
+int or_synth_gemv_threads(const or_factors *f, const or_schedule *s, int64_t tie_count,
+                          uint64_t key, const uint32_t *taps, int nb,
+                          const uint16_t *x_bf16, int64_t r0, int64_t nrows, double *y,
+                          double *yabs, int nthreads);
+
+/* Pack rows [r0, r0+nrows) of the synthetic stream at bit 0 of out (zeroed by
+ * the caller); returns the bits written. */
+uint64_t or_synth_pack_rows(const or_factors *f, const or_schedule *s, int64_t tie_count,
+                            uint64_t key, int64_t r0, int64_t nrows, uint8_t *out);
 
 /* ---------------- encoder side (Sec. 3.4, App. A.5, Eq. codec search) ------ */
 

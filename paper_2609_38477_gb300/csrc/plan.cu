@@ -1,0 +1,565 @@
+// Decoder plan of Alg. 2 (imp, floor, ladder, tie pass, row offsets), LFSR jump
+// tables, layer lifetime and the synthetic stream generator.
+#include <cuda_fp16.h>
+#include <math.h>
+#include <stdio.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include "seedq_internal.cuh"
+
+namespace seedq {
+
+static thread_local char g_last_cuda_error[256] = "";
+
+seedq_status cuda_fail(cudaError_t e) {
+  snprintf(g_last_cuda_error, sizeof g_last_cuda_error, "%s: %s", cudaGetErrorName(e),
+           cudaGetErrorString(e));
+  return SEEDQ_ERR_CUDA;
+}
+
+// Feedback taps of the width-S LFSR of the stream format: o_{t+S} = XOR over
+// set bits i of o_{t+i}.  Each is a primitive polynomial x^S + sum x^i with the
+// smallest possible largest tap below S (so one machine word yields the most
+// new sequence bits per step), then the fewest taps, then the smallest mask.
+static const uint32_t kTaps[17] = {0, 0, 0, 0, 0, 0, 0, 0,
+                                   0x1d,  // S=8:  x^8+x^4+x^3+x^2+1
+                                   0x11,  // S=9:  x^9+x^4+1
+                                   0x09,  // S=10: x^10+x^3+1
+                                   0x05,  // S=11: x^11+x^2+1
+                                   0x53,  // S=12: x^12+x^6+x^4+x+1
+                                   0x1b,  // S=13: x^13+x^4+x^3+x+1
+                                   0x2b,  // S=14: x^14+x^5+x^3+x+1
+                                   0x03,  // S=15: x^15+x+1
+                                   0x2d}; // S=16: x^16+x^5+x^3+x^2+1
+
+// ------------------------------------------------------------ plan kernels
+
+// Stable ascending rank of a: perm[rank(i)] = i with ties broken by index
+// (Sec. 3.3: channels sorted by a before blocking).
+__global__ void k_perm(const float *__restrict__ a, int C, int32_t *__restrict__ perm) {
+  __shared__ float tile[1024];
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  const float ai = (i < C) ? a[i] : 0.f;
+  int rank = 0;
+  for (int base = 0; base < C; base += 1024) {
+    __syncthreads();
+    for (int t = threadIdx.x; t < 1024; t += blockDim.x)
+      tile[t] = (base + t < C) ? a[base + t] : 0.f;
+    __syncthreads();
+    const int n = min(1024, C - base);
+    for (int t = 0; t < n; ++t) {
+      const float v = tile[t];
+      rank += (v < ai || (v == ai && base + t < i)) ? 1 : 0;
+    }
+  }
+  if (i < C) perm[rank] = i;
+}
+
+// Block means of the permuted a, summed in channel order, and their unit-mean
+// normalization summed in ascending block order (Eq. imp; App. A.7 fixed order).
+__global__ void k_abar(const float *__restrict__ a, const int32_t *__restrict__ perm,
+                       int nb, double *__restrict__ abar) {
+  __shared__ double mean;
+  for (int c = threadIdx.x; c < nb; c += blockDim.x) {
+    double s = 0.0;
+    for (int i = 0; i < 8; ++i) s = __dadd_rn(s, (double)a[perm[8 * c + i]]);
+    abar[c] = __ddiv_rn(s, 8.0);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double s = 0.0;
+    for (int c = 0; c < nb; ++c) s = __dadd_rn(s, abar[c]);
+    mean = __ddiv_rn(s, (double)nb);
+  }
+  __syncthreads();
+  for (int c = threadIdx.x; c < nb; c += blockDim.x) abar[c] = __ddiv_rn(abar[c], mean);
+}
+
+// Row factor normalized to unit mean, summed in ascending row order.
+__global__ void k_rho(const float *__restrict__ rho_in, int64_t R, double *__restrict__ rho) {
+  __shared__ double mean;
+  if (threadIdx.x == 0) {
+    double s = 0.0;
+    if (rho_in)
+      for (int64_t r = 0; r < R; ++r) s = __dadd_rn(s, (double)rho_in[r]);
+    mean = __ddiv_rn(s, (double)R);
+  }
+  __syncthreads();
+  for (int64_t r = threadIdx.x; r < R; r += blockDim.x)
+    rho[r] = rho_in ? __ddiv_rn((double)rho_in[r], mean) : 1.0;
+}
+
+struct SchedArgs {
+  int J;
+  int j_tie;
+  double q;
+  double theta[kMaxJ];
+};
+
+// Floored importance of block c of a row with factor rr: max(abar_c * rho_r, q).
+__device__ __forceinline__ double imp_at(const double *abar, double rr, double q, int c) {
+  const double v = __dmul_rn(abar[c], rr);
+  return (v < q) ? q : v;
+}
+
+// First block of the row whose importance is >= thr (> thr when strict);
+// importance is non-decreasing along a row because channels are sorted.
+__device__ int first_block(const double *abar, double rr, double q, int nb, double thr,
+                           bool strict) {
+  int lo = 0, hi = nb;
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    const double v = imp_at(abar, rr, q, mid);
+    const bool pass = strict ? (v > thr) : (v >= thr);
+    if (pass) hi = mid;
+    else lo = mid + 1;
+  }
+  return lo;
+}
+
+// Eq. ladder as breakpoints: brk[r][j] = first block with theta_j <= imp, i.e.
+// rung >= j+1; tcnt[r] = blocks of the row tied at theta[j_tie].
+__global__ void k_rows(const double *__restrict__ abar, const double *__restrict__ rho,
+                       int nb, int64_t R, SchedArgs s, int32_t *__restrict__ brk,
+                       int32_t *__restrict__ tcnt) {
+  const int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= R) return;
+  const double rr = rho[r];
+  for (int j = 0; j < s.J - 1; ++j)
+    brk[r * (s.J - 1) + j] = first_block(abar, rr, s.q, nb, s.theta[j], false);
+  int t = 0;
+  if (s.j_tie >= 0) {
+    const int hi = first_block(abar, rr, s.q, nb, s.theta[s.j_tie], true);
+    t = hi - brk[r * (s.J - 1) + s.j_tie];
+  }
+  tcnt[r] = t;
+}
+
+// Block-wide exclusive scan of per-thread totals (1024 threads).
+__device__ uint64_t block_exclusive_scan(uint64_t v, uint64_t *sh, uint64_t *total) {
+  const int t = threadIdx.x;
+  sh[t] = v;
+  __syncthreads();
+  for (int d = 1; d < blockDim.x; d <<= 1) {
+    const uint64_t add = (t >= d) ? sh[t - d] : 0;
+    __syncthreads();
+    sh[t] += add;
+    __syncthreads();
+  }
+  const uint64_t incl = sh[t];
+  if (total) *total = sh[blockDim.x - 1];
+  __syncthreads();
+  return incl - v;
+}
+
+// Tie pass of Alg. 2 (the first T tied blocks in row-major order take the lower
+// rung) applied to the breakpoints, then per-row bit counts and their exclusive
+// scan into row offsets.  One CTA of 1024 threads, rows in contiguous chunks.
+__global__ void k_scan(int64_t R, int J, int nb, int j_tie, int64_t T, const int *Lrung,
+                       int32_t *__restrict__ brk, const int32_t *__restrict__ tcnt,
+                       uint64_t *__restrict__ row_off, uint64_t *__restrict__ summary) {
+  __shared__ uint64_t sh[1024];
+  __shared__ int L[kMaxJ];
+  if (threadIdx.x < J) L[threadIdx.x] = Lrung[threadIdx.x];
+  const int64_t per = (R + blockDim.x - 1) / blockDim.x;
+  const int64_t r0 = min((int64_t)threadIdx.x * per, R), r1 = min(r0 + per, R);
+  uint64_t tied_total = 0;
+  if (j_tie >= 0) {
+    uint64_t local = 0;
+    for (int64_t r = r0; r < r1; ++r) local += (uint64_t)tcnt[r];
+    uint64_t prefix = block_exclusive_scan(local, sh, &tied_total);
+    for (int64_t r = r0; r < r1; ++r) {
+      const int64_t left = T - (int64_t)prefix;
+      const int64_t d = left <= 0 ? 0 : (left < tcnt[r] ? left : tcnt[r]);
+      brk[r * (J - 1) + j_tie] += (int32_t)d;
+      prefix += (uint64_t)tcnt[r];
+    }
+  }
+  __syncthreads();
+  uint64_t local = 0;
+  for (int64_t r = r0; r < r1; ++r) {
+    uint64_t b = (uint64_t)L[0] * (uint64_t)nb;
+    for (int j = 0; j < J - 1; ++j)
+      b += (uint64_t)(L[j + 1] - L[j]) * (uint64_t)(nb - brk[r * (J - 1) + j]);
+    local += b;
+  }
+  uint64_t total = 0;
+  uint64_t off = block_exclusive_scan(local, sh, &total);
+  for (int64_t r = r0; r < r1; ++r) {
+    row_off[r] = off;
+    uint64_t b = (uint64_t)L[0] * (uint64_t)nb;
+    for (int j = 0; j < J - 1; ++j)
+      b += (uint64_t)(L[j + 1] - L[j]) * (uint64_t)(nb - brk[r * (J - 1) + j]);
+    off += b;
+  }
+  if (threadIdx.x == 0) {
+    row_off[R] = total;
+    summary[0] = tied_total;
+    summary[1] = total;
+  }
+}
+
+// GF(2) jump tables: tab[v] = first 64 sequence bits from seed v, tab[256+v]
+// from seed v << 8; by linearity the prefix of any seed is the XOR of the two.
+__global__ void k_tables(const int32_t *__restrict__ slot_S, uint64_t *__restrict__ tables,
+                         uint32_t t0, uint32_t t1, uint32_t t2, uint32_t t3, uint32_t t4,
+                         uint32_t t5, uint32_t t6, uint32_t t7, uint32_t t8) {
+  const uint32_t taps_arr[9] = {t0, t1, t2, t3, t4, t5, t6, t7, t8};
+  const int slot = blockIdx.x;
+  const int S = slot_S[slot];
+  const uint32_t taps = taps_arr[S - 8];
+  const int v = threadIdx.x;  // 0..511
+  const uint32_t seed = (v < 256) ? (uint32_t)v : ((uint32_t)(v - 256) << 8);
+  uint64_t q = (uint64_t)(seed & ((1u << S) - 1u));
+  if (v >= 256 && S <= 8) q = 0;
+  for (int t = S; t < 64; ++t) {
+    const uint64_t win = (q >> (t - S)) & (uint64_t)taps;
+    const uint64_t bit = (uint64_t)(__popcll(win) & 1);
+    q |= bit << t;
+  }
+  tables[(size_t)slot * 512 + v] = q;
+}
+
+// Synthetic payload of the workload recipe, one thread per block.
+__device__ __forceinline__ uint64_t splitmix64_at(uint64_t key, uint64_t i) {
+  uint64_t z = key + (i + 1ull) * 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+__global__ void k_synth(const __grid_constant__ LayerArgs p, const int32_t *__restrict__ S_of, const int32_t *__restrict__ K_of,
+                        uint64_t key, uint32_t *__restrict__ out) {
+  const int64_t total = p.R * (int64_t)p.nb;
+  for (int64_t b = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; b < total;
+       b += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t r = b / p.nb;
+    const int c = (int)(b - r * p.nb);
+    int32_t bk[kMaxJ];
+    for (int j = 0; j < p.J - 1; ++j) bk[j] = p.brk[r * (p.J - 1) + j];
+    const int g = rung_of(bk, p.J, c);
+    const int S = S_of[g], K = K_of[g];
+    const uint64_t off = p.row_off[r] + bits_before(bk, p.J, p.L, p.nb, c);
+    const uint64_t h = splitmix64_at(key, (uint64_t)b);
+    const uint32_t seed = 1u + (uint32_t)(h >> 32) % ((1u << S) - 1u);
+    const int E = -8 + (int)(((h >> 24) & 255u) % 6u);
+    uint64_t v = (uint64_t)seed | ((uint64_t)(E & 15) << S);
+    for (int j = 0; j < K; ++j) {
+      const int t = (int)((h >> (4 * j)) & 15u) - 8;
+      v |= (uint64_t)(t & 15) << (S + 4 + 4 * j);
+    }
+    const uint64_t wi = off >> 5;
+    const int sh = (int)(off & 31);
+    atomicOr(out + wi, (uint32_t)(v << sh));
+    const uint64_t rest = (sh == 0) ? (v >> 32) : (v >> (32 - sh));
+    if (rest) atomicOr(out + wi + 1, (uint32_t)rest);
+    const uint64_t rest2 = (sh == 0) ? 0 : (v >> (64 - sh));
+    if (sh && rest2) atomicOr(out + wi + 2, (uint32_t)rest2);
+  }
+}
+
+static void free_layer(seedq_layer *L) {
+  if (!L) return;
+  cudaFree(L->d_perm);
+  cudaFree(L->d_abar);
+  cudaFree(L->d_rho);
+  cudaFree(L->d_rho_in);
+  cudaFree(L->d_a_in);
+  cudaFree(L->d_brk);
+  cudaFree(L->d_tcnt);
+  cudaFree(L->d_row_off);
+  cudaFree(L->d_tables);
+  cudaFree(L->d_flags);
+  cudaFree(L->d_summary);
+  cudaFree(L->d_partials);
+  free(L);
+}
+
+int64_t gemv_partial_elems(const seedq_layer *L, int max_batch);  // gemv.cu
+
+}  // namespace seedq
+
+using namespace seedq;
+
+extern "C" {
+
+const char *seedq_status_string(seedq_status s) {
+  switch (s) {
+    case SEEDQ_OK: return "ok";
+    case SEEDQ_ERR_INVALID_ARG: return "invalid argument";
+    case SEEDQ_ERR_STREAM: return "stream length or buffer size does not match the plan";
+    case SEEDQ_ERR_SCHEDULE: return "inconsistent schedule tables";
+    case SEEDQ_ERR_CUDA: return "CUDA error";
+    case SEEDQ_ERR_NOMEM: return "out of memory";
+    case SEEDQ_ERR_UNSUPPORTED: return "unsupported rung or shape";
+  }
+  return "unknown status";
+}
+
+const char *seedq_last_cuda_error_string(void) { return g_last_cuda_error; }
+
+uint32_t seedq_lfsr_taps(int32_t S) { return (S >= 8 && S <= 16) ? kTaps[S] : 0u; }
+
+uint64_t seedq_stream_bytes_required(uint64_t bits) { return stream_bytes_required(bits); }
+
+seedq_status seedq_layer_prepare(const seedq_layer_desc *d, const seedq_schedule *s,
+                                 void *cuda_stream, seedq_layer **out) {
+  if (!d || !s || !out) return SEEDQ_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (d->rows < 1 || d->rows > (1ll << 24) || d->cols < 8 || (d->cols % 8) != 0 || !d->a)
+    return SEEDQ_ERR_INVALID_ARG;
+  if (d->cols > kMaxCols) return SEEDQ_ERR_UNSUPPORTED;
+  if (d->n_outliers < 0 || d->n_outliers > kMaxOutliers) return SEEDQ_ERR_INVALID_ARG;
+  if (d->n_outliers > 0 && (!d->outlier_cols || !d->outlier_vals)) return SEEDQ_ERR_INVALID_ARG;
+  if (d->tie_count < 0) return SEEDQ_ERR_SCHEDULE;
+  const int mb = d->max_batch == 0 ? kMaxBatch : d->max_batch;
+  if (mb < 1 || mb > kMaxBatch) return SEEDQ_ERR_INVALID_ARG;
+  if (s->J < 1 || s->J > kMaxJ || !s->rungs || (s->J > 1 && !s->theta)) return SEEDQ_ERR_SCHEDULE;
+  for (int j = 0; j < s->J; ++j) {
+    if (!rung_supported(s->rungs[j].S, s->rungs[j].k)) return SEEDQ_ERR_UNSUPPORTED;
+    if (j > 0 && s->rungs[j].S + 4 * s->rungs[j].k <= s->rungs[j - 1].S + 4 * s->rungs[j - 1].k)
+      return SEEDQ_ERR_SCHEDULE;
+  }
+  for (int j = 0; j + 1 < s->J; ++j) {
+    if (!isfinite(s->theta[j])) return SEEDQ_ERR_SCHEDULE;
+    if (j > 0 && !(s->theta[j] > s->theta[j - 1])) return SEEDQ_ERR_SCHEDULE;
+  }
+  if (s->j_tie < -1 || s->j_tie >= s->J - 1 || (s->J == 1 && s->j_tie != -1)) return SEEDQ_ERR_SCHEDULE;
+  if (!isfinite(s->q)) return SEEDQ_ERR_SCHEDULE;
+  double asum = 0.0;
+  for (int64_t c = 0; c < d->cols; ++c) {
+    if (!isfinite(d->a[c]) || d->a[c] < 0.f) return SEEDQ_ERR_INVALID_ARG;
+    asum += d->a[c];
+  }
+  if (!(asum > 0.0)) return SEEDQ_ERR_INVALID_ARG;
+  if (d->rho)
+    for (int64_t r = 0; r < d->rows; ++r)
+      if (!isfinite(d->rho[r]) || !(d->rho[r] > 0.f)) return SEEDQ_ERR_INVALID_ARG;
+  for (int o = 0; o < d->n_outliers; ++o) {
+    if (d->outlier_cols[o] < 0 || d->outlier_cols[o] >= d->cols) return SEEDQ_ERR_INVALID_ARG;
+    for (int p = 0; p < o; ++p)
+      if (d->outlier_cols[p] == d->outlier_cols[o]) return SEEDQ_ERR_INVALID_ARG;
+  }
+
+  seedq_layer *L = (seedq_layer *)calloc(1, sizeof(seedq_layer));
+  if (!L) return SEEDQ_ERR_NOMEM;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  const int64_t R = d->rows, C = d->cols;
+  const int nb = (int)(C / 8), J = s->J;
+  L->args.R = R;
+  L->args.C = C;
+  L->args.nb = nb;
+  L->args.J = J;
+  L->j_tie = s->j_tie;
+  L->q = s->q;
+  L->tie_count = d->tie_count;
+  L->max_batch = mb;
+  cudaGetDevice(&L->device);
+  int nslots = 0;
+  for (int j = 0; j < J; ++j) {
+    L->S[j] = s->rungs[j].S;
+    L->k[j] = s->rungs[j].k;
+    L->args.L[j] = L->S[j] + 4 * L->k[j] + 4;
+    L->args.code[j] = rung_code(L->S[j], L->k[j]);
+    int slot = -1;
+    for (int t = 0; t < nslots; ++t)
+      if (L->slot_S[t] == L->S[j]) slot = t;
+    if (slot < 0) {
+      slot = nslots;
+      L->slot_S[nslots++] = L->S[j];
+    }
+    L->args.slot[j] = slot;
+    if (j + 1 < J) L->theta[j] = s->theta[j];
+  }
+  L->args.nslots = nslots;
+  L->args.n_out = d->n_outliers;
+  for (int o = 0; o < d->n_outliers; ++o) L->args.out_cols[o] = d->outlier_cols[o];
+  L->args.out_vals = d->outlier_vals;
+
+  const int Jm1 = J > 1 ? J - 1 : 1;
+  seedq_status rc = SEEDQ_OK;
+#define ALLOC(ptr, bytes)                                              \
+  do {                                                                 \
+    cudaError_t e_ = cudaMalloc((void **)&(ptr), (bytes));             \
+    if (e_ != cudaSuccess) {                                           \
+      cudaGetLastError();                                              \
+      free_layer(L);                                                   \
+      return e_ == cudaErrorMemoryAllocation ? SEEDQ_ERR_NOMEM : cuda_fail(e_); \
+    }                                                                  \
+  } while (0)
+  ALLOC(L->d_perm, sizeof(int32_t) * C);
+  ALLOC(L->d_abar, sizeof(double) * nb);
+  ALLOC(L->d_rho, sizeof(double) * R);
+  ALLOC(L->d_a_in, sizeof(float) * C);
+  if (d->rho) ALLOC(L->d_rho_in, sizeof(float) * R);
+  ALLOC(L->d_brk, sizeof(int32_t) * R * Jm1);
+  ALLOC(L->d_tcnt, sizeof(int32_t) * R);
+  ALLOC(L->d_row_off, sizeof(uint64_t) * (R + 1));
+  ALLOC(L->d_tables, sizeof(uint64_t) * 512 * nslots);
+  ALLOC(L->d_flags, sizeof(uint32_t));
+  ALLOC(L->d_summary, sizeof(uint64_t) * 2);
+  {
+    int32_t *dS = nullptr;
+    ALLOC(dS, sizeof(int32_t) * kMaxJ);
+    cudaError_t e = cudaMemcpyAsync(dS, L->slot_S, sizeof(int32_t) * kMaxJ, cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess) {
+      k_tables<<<nslots, 512, 0, st>>>(dS, L->d_tables, kTaps[8], kTaps[9], kTaps[10], kTaps[11],
+                                       kTaps[12], kTaps[13], kTaps[14], kTaps[15], kTaps[16]);
+      e = cudaGetLastError();
+    }
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    cudaFree(dS);
+    if (e != cudaSuccess) { free_layer(L); return cuda_fail(e); }
+  }
+  L->partial_elems = gemv_partial_elems(L, mb);
+  if (L->partial_elems) ALLOC(L->d_partials, sizeof(float) * L->partial_elems);
+#undef ALLOC
+  L->args.perm = L->d_perm;
+  L->args.brk = L->d_brk;
+  L->args.row_off = L->d_row_off;
+  L->args.tables = L->d_tables;
+  L->args.flags = L->d_flags;
+  L->args.stream = nullptr;
+
+  int *dL = nullptr;
+  cudaError_t e = cudaMalloc((void **)&dL, sizeof(int) * kMaxJ);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(dL, L->args.L, sizeof(int) * kMaxJ, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(L->d_flags, 0, sizeof(uint32_t), st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(L->d_a_in, d->a, sizeof(float) * C, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess && d->rho)
+    e = cudaMemcpyAsync(L->d_rho_in, d->rho, sizeof(float) * R, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) {
+    k_perm<<<(int)((C + 255) / 256), 256, 0, st>>>(L->d_a_in, (int)C, L->d_perm);
+    k_abar<<<1, 1024, 0, st>>>(L->d_a_in, L->d_perm, nb, L->d_abar);
+    k_rho<<<1, 1024, 0, st>>>(L->d_rho_in, R, L->d_rho);
+    SchedArgs sa;
+    sa.J = J;
+    sa.j_tie = s->j_tie;
+    sa.q = s->q;
+    for (int j = 0; j < kMaxJ; ++j) sa.theta[j] = (j + 1 < J) ? s->theta[j] : 0.0;
+    if (J > 1) {
+      k_rows<<<(int)((R + 255) / 256), 256, 0, st>>>(L->d_abar, L->d_rho, nb, R, sa, L->d_brk,
+                                                     L->d_tcnt);
+    } else {
+      e = cudaMemsetAsync(L->d_tcnt, 0, sizeof(int32_t) * R, st);
+    }
+    k_scan<<<1, 1024, 0, st>>>(R, J, nb, J > 1 ? s->j_tie : -1, d->tie_count, dL, L->d_brk,
+                               L->d_tcnt, L->d_row_off, L->d_summary);
+    if (e == cudaSuccess) e = cudaGetLastError();
+  }
+  uint64_t summary[2] = {0, 0};
+  if (e == cudaSuccess) e = cudaMemcpyAsync(summary, L->d_summary, sizeof summary, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  cudaFree(dL);
+  if (e != cudaSuccess) {
+    free_layer(L);
+    return cuda_fail(e);
+  }
+  if (s->j_tie >= 0 && (uint64_t)d->tie_count > summary[0]) rc = SEEDQ_ERR_SCHEDULE;
+  if (s->j_tie < 0 && d->tie_count != 0) rc = SEEDQ_ERR_SCHEDULE;
+  if (rc != SEEDQ_OK) {
+    free_layer(L);
+    return rc;
+  }
+  L->total_bits = summary[1];
+  // The plan's fp32 copies of a and rho are no longer needed.
+  cudaFree(L->d_a_in);
+  L->d_a_in = nullptr;
+  cudaFree(L->d_rho_in);
+  L->d_rho_in = nullptr;
+  *out = L;
+  return SEEDQ_OK;
+}
+
+seedq_status seedq_layer_stream_bits(const seedq_layer *L, uint64_t *bits) {
+  if (!L || !bits) return SEEDQ_ERR_INVALID_ARG;
+  *bits = L->total_bits;
+  return SEEDQ_OK;
+}
+
+seedq_status seedq_layer_bind_stream(seedq_layer *L, const void *stream, uint64_t bits,
+                                     uint64_t bytes) {
+  if (!L || !stream) return SEEDQ_ERR_INVALID_ARG;
+  if (((uintptr_t)stream & 15u) != 0) return SEEDQ_ERR_INVALID_ARG;
+  if (bits != L->total_bits || bytes < stream_bytes_required(bits)) return SEEDQ_ERR_STREAM;
+  L->stream = stream;
+  L->stream_bytes = bytes;
+  L->args.stream = (const uint32_t *)stream;
+  return SEEDQ_OK;
+}
+
+seedq_status seedq_layer_release(seedq_layer *L) {
+  if (!L) return SEEDQ_OK;
+  cudaError_t e = cudaDeviceSynchronize();
+  free_layer(L);
+  return e == cudaSuccess ? SEEDQ_OK : cuda_fail(e);
+}
+
+seedq_status seedq_layer_rung_map(const seedq_layer *L, int64_t row0, int64_t nrows,
+                                  uint8_t *rungs_host) {
+  if (!L || !rungs_host || row0 < 0 || nrows < 0 || row0 + nrows > L->args.R)
+    return SEEDQ_ERR_INVALID_ARG;
+  const int J = L->args.J, nb = L->args.nb, Jm1 = J > 1 ? J - 1 : 1;
+  int32_t *bk = (int32_t *)malloc(sizeof(int32_t) * (size_t)(nrows * Jm1 + 1));
+  if (!bk) return SEEDQ_ERR_NOMEM;
+  if (nrows) {
+    cudaError_t e = cudaMemcpy(bk, L->d_brk + row0 * Jm1, sizeof(int32_t) * nrows * Jm1,
+                               cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) { free(bk); return cuda_fail(e); }
+  }
+  for (int64_t i = 0; i < nrows; ++i)
+    for (int c = 0; c < nb; ++c) {
+      int j = 0;
+      for (int t = 0; t < J - 1; ++t) j += (bk[i * Jm1 + t] <= c) ? 1 : 0;
+      rungs_host[i * nb + c] = (uint8_t)j;
+    }
+  free(bk);
+  return SEEDQ_OK;
+}
+
+seedq_status seedq_layer_perm(const seedq_layer *L, int32_t *perm_host) {
+  if (!L || !perm_host) return SEEDQ_ERR_INVALID_ARG;
+  SEEDQ_CUDA(cudaMemcpy(perm_host, L->d_perm, sizeof(int32_t) * L->args.C, cudaMemcpyDeviceToHost));
+  return SEEDQ_OK;
+}
+
+seedq_status seedq_layer_row_offsets(const seedq_layer *L, uint64_t *offs) {
+  if (!L || !offs) return SEEDQ_ERR_INVALID_ARG;
+  SEEDQ_CUDA(cudaMemcpy(offs, L->d_row_off, sizeof(uint64_t) * (L->args.R + 1), cudaMemcpyDeviceToHost));
+  return SEEDQ_OK;
+}
+
+seedq_status seedq_last_device_error(const seedq_layer *L, uint32_t *flags) {
+  if (!L || !flags) return SEEDQ_ERR_INVALID_ARG;
+  SEEDQ_CUDA(cudaMemcpy(flags, L->d_flags, sizeof(uint32_t), cudaMemcpyDeviceToHost));
+  return SEEDQ_OK;
+}
+
+seedq_status seedq_synth_stream(const seedq_layer *L, uint64_t key, void *stream,
+                                uint64_t stream_bytes, void *cuda_stream) {
+  if (!L || !stream || ((uintptr_t)stream & 15u)) return SEEDQ_ERR_INVALID_ARG;
+  if (stream_bytes < stream_bytes_required(L->total_bits)) return SEEDQ_ERR_STREAM;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  int32_t *dSK = nullptr;
+  SEEDQ_CUDA(cudaMalloc((void **)&dSK, sizeof(int32_t) * 2 * kMaxJ));
+  int32_t hSK[2 * kMaxJ];
+  for (int j = 0; j < kMaxJ; ++j) {
+    hSK[j] = L->S[j];
+    hSK[kMaxJ + j] = L->k[j];
+  }
+  cudaError_t e = cudaMemcpyAsync(dSK, hSK, sizeof hSK, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(stream, 0, stream_bytes, st);
+  if (e == cudaSuccess) {
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    k_synth<<<sms * 8, 256, 0, st>>>(L->args, dSK, dSK + kMaxJ, key, (uint32_t *)stream);
+    e = cudaGetLastError();
+  }
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  cudaFree(dSK);
+  return e == cudaSuccess ? SEEDQ_OK : cuda_fail(e);
+}
+
+}  // extern "C"

@@ -1,0 +1,210 @@
+"""Python binding of libseedq.so: argument marshalling only.
+
+Every function forwards to the C ABI declared in include/seedq.h under the same
+name; all computation happens in the library's CUDA kernels.  Device buffers
+are passed as torch tensors (their data_ptr) or raw integer addresses, and the
+CUDA stream as torch.cuda.Stream / raw handle / None (torch's current stream).
+If the library is missing this module raises at import of the handle: there is
+no fallback path.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libseedq.so")
+_lib = None
+
+STATUS = {0: "SEEDQ_OK", 1: "SEEDQ_ERR_INVALID_ARG", 2: "SEEDQ_ERR_STREAM",
+          3: "SEEDQ_ERR_SCHEDULE", 4: "SEEDQ_ERR_CUDA", 5: "SEEDQ_ERR_NOMEM",
+          6: "SEEDQ_ERR_UNSUPPORTED"}
+
+
+class SeedQError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        msg = lib().seedq_status_string(status).decode()
+        if status == 4:
+            msg += ": " + lib().seedq_last_cuda_error_string().decode()
+        super().__init__(f"{where}: {STATUS.get(status, status)} ({msg})")
+        self.status = status
+
+
+class Rung(C.Structure):
+    _fields_ = [("S", C.c_int32), ("k", C.c_int32)]
+
+
+class Schedule(C.Structure):
+    _fields_ = [("J", C.c_int32), ("rungs", C.POINTER(Rung)), ("theta", C.POINTER(C.c_double)),
+                ("j_tie", C.c_int32), ("q", C.c_double)]
+
+
+class LayerDesc(C.Structure):
+    _fields_ = [("rows", C.c_int64), ("cols", C.c_int64), ("a", C.POINTER(C.c_float)),
+                ("rho", C.POINTER(C.c_float)), ("tie_count", C.c_int64),
+                ("n_outliers", C.c_int32), ("outlier_cols", C.POINTER(C.c_int32)),
+                ("outlier_vals", C.c_void_p), ("max_batch", C.c_int32)]
+
+
+# Every symbol include/seedq.h declares, with its ctypes signature.
+SIGNATURES = {
+    "seedq_layer_prepare": (C.c_int, [C.POINTER(LayerDesc), C.POINTER(Schedule), C.c_void_p,
+                                      C.POINTER(C.c_void_p)]),
+    "seedq_layer_stream_bits": (C.c_int, [C.c_void_p, C.POINTER(C.c_uint64)]),
+    "seedq_stream_bytes_required": (C.c_uint64, [C.c_uint64]),
+    "seedq_layer_bind_stream": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint64, C.c_uint64]),
+    "seedq_layer_release": (C.c_int, [C.c_void_p]),
+    "seedq_decode_weights": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
+    "seedq_decode_rows": (C.c_int, [C.c_void_p, C.c_int64, C.c_int64, C.c_void_p, C.c_void_p]),
+    "seedq_gemv": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
+    "seedq_gemm_small_batch": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p]),
+    "seedq_layer_rung_map": (C.c_int, [C.c_void_p, C.c_int64, C.c_int64, C.c_void_p]),
+    "seedq_layer_perm": (C.c_int, [C.c_void_p, C.c_void_p]),
+    "seedq_layer_row_offsets": (C.c_int, [C.c_void_p, C.c_void_p]),
+    "seedq_last_device_error": (C.c_int, [C.c_void_p, C.POINTER(C.c_uint32)]),
+    "seedq_lfsr_taps": (C.c_uint32, [C.c_int32]),
+    "seedq_synth_stream": (C.c_int, [C.c_void_p, C.c_uint64, C.c_void_p, C.c_uint64, C.c_void_p]),
+    "seedq_status_string": (C.c_char_p, [C.c_int]),
+    "seedq_last_cuda_error_string": (C.c_char_p, []),
+}
+
+
+def lib():
+    """The loaded libseedq.so (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise ImportError(f"{LIB_PATH} is missing: run __graft_entry__.build() "
+                              "(there is no CPU fallback)")
+        L = C.CDLL(LIB_PATH)
+        for name, (res, args) in SIGNATURES.items():
+            fn = getattr(L, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = L
+    return _lib
+
+
+def _check(status: int, where: str):
+    if status != 0:
+        raise SeedQError(status, where)
+
+
+def _ptr(t) -> int:
+    if t is None:
+        return 0
+    if isinstance(t, int):
+        return t
+    return t.data_ptr()
+
+
+def _stream(s) -> int:
+    if s is None:
+        import torch
+
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(s, int):
+        return s
+    return s.cuda_stream
+
+
+def stream_bytes_required(bits: int) -> int:
+    return lib().seedq_stream_bytes_required(bits)
+
+
+def lfsr_taps(S: int) -> int:
+    return lib().seedq_lfsr_taps(S)
+
+
+class Layer:
+    """One prepared tensor (seedq_layer_prepare ... seedq_layer_release)."""
+
+    def __init__(self, rows, cols, a, rho, rungs, theta, j_tie, q, tie_count,
+                 outlier_cols=None, outlier_vals=None, max_batch=0, stream=None):
+        self.rows, self.cols = int(rows), int(cols)
+        self._a = np.ascontiguousarray(a, np.float32)
+        self._rho = None if rho is None else np.ascontiguousarray(rho, np.float32)
+        self._rungs = (Rung * len(rungs))(*[Rung(int(S), int(k)) for S, k in rungs])
+        self._theta = np.ascontiguousarray(theta, np.float64)
+        if self._theta.size == 0:
+            self._theta = np.zeros(1, np.float64)
+        self._ocols = (np.zeros(1, np.int32) if outlier_cols is None
+                       else np.ascontiguousarray(outlier_cols, np.int32))
+        self._ovals = outlier_vals  # device tensor, kept alive with the layer
+        n_out = 0 if outlier_cols is None else len(outlier_cols)
+        desc = LayerDesc(self.rows, self.cols, self._a.ctypes.data_as(C.POINTER(C.c_float)),
+                         None if self._rho is None else self._rho.ctypes.data_as(C.POINTER(C.c_float)),
+                         int(tie_count), n_out, self._ocols.ctypes.data_as(C.POINTER(C.c_int32)),
+                         _ptr(outlier_vals), int(max_batch))
+        sched = Schedule(len(rungs), self._rungs, self._theta.ctypes.data_as(C.POINTER(C.c_double)),
+                         int(j_tie), float(q))
+        h = C.c_void_p()
+        _check(lib().seedq_layer_prepare(C.byref(desc), C.byref(sched), _stream(stream), C.byref(h)),
+               "seedq_layer_prepare")
+        self.h = h
+        self._stream_buf = None
+
+    # -- lifetime ---------------------------------------------------------
+    def release(self):
+        if self.h is not None and self.h.value:
+            _check(lib().seedq_layer_release(self.h), "seedq_layer_release")
+        self.h = None
+
+    def __del__(self):
+        try:
+            self.release()
+        except Exception:
+            pass
+
+    # -- stream -----------------------------------------------------------
+    @property
+    def stream_bits(self) -> int:
+        b = C.c_uint64()
+        _check(lib().seedq_layer_stream_bits(self.h, C.byref(b)), "seedq_layer_stream_bits")
+        return b.value
+
+    def bind_stream(self, buf, bits: int, nbytes: int):
+        _check(lib().seedq_layer_bind_stream(self.h, _ptr(buf), bits, nbytes), "seedq_layer_bind_stream")
+        self._stream_buf = buf
+
+    def synth_stream(self, key: int, buf, nbytes: int, stream=None):
+        _check(lib().seedq_synth_stream(self.h, key, _ptr(buf), nbytes, _stream(stream)),
+               "seedq_synth_stream")
+
+    # -- hot calls --------------------------------------------------------
+    def decode_weights(self, W, stream=None):
+        _check(lib().seedq_decode_weights(self.h, _ptr(W), _stream(stream)), "seedq_decode_weights")
+
+    def decode_rows(self, row0: int, nrows: int, W, stream=None):
+        _check(lib().seedq_decode_rows(self.h, row0, nrows, _ptr(W), _stream(stream)), "seedq_decode_rows")
+
+    def gemv(self, x, y, stream=None):
+        _check(lib().seedq_gemv(self.h, _ptr(x), _ptr(y), _stream(stream)), "seedq_gemv")
+
+    def gemm_small_batch(self, X, n: int, Y, stream=None):
+        _check(lib().seedq_gemm_small_batch(self.h, _ptr(X), n, _ptr(Y), _stream(stream)),
+               "seedq_gemm_small_batch")
+
+    # -- introspection (synchronous) --------------------------------------
+    def rung_map(self, row0: int = 0, nrows: int | None = None) -> np.ndarray:
+        nrows = self.rows - row0 if nrows is None else nrows
+        out = np.zeros((nrows, self.cols // 8), np.uint8)
+        _check(lib().seedq_layer_rung_map(self.h, row0, nrows, out.ctypes.data), "seedq_layer_rung_map")
+        return out
+
+    def perm(self) -> np.ndarray:
+        out = np.zeros(self.cols, np.int32)
+        _check(lib().seedq_layer_perm(self.h, out.ctypes.data), "seedq_layer_perm")
+        return out
+
+    def row_offsets(self) -> np.ndarray:
+        out = np.zeros(self.rows + 1, np.uint64)
+        _check(lib().seedq_layer_row_offsets(self.h, out.ctypes.data), "seedq_layer_row_offsets")
+        return out
+
+    def device_error(self) -> int:
+        f = C.c_uint32()
+        _check(lib().seedq_last_device_error(self.h, C.byref(f)), "seedq_last_device_error")
+        return f.value
