@@ -380,8 +380,6 @@ def our_arm(args):
     hbm_peak = (peaks or {}).get("hbm_gbs") or 6800.0
     achieved_issue = warp_inst / (kern_ms * 1e-3) / 1e9
     achieved_hbm = alg_bytes / (kern_ms * 1e-3) / 1e9
-    nbt = 1 if n <= 1 else 2 if n <= 2 else 4 if n <= 4 else 8 if n <= 8 else 16
-    nsplit_tensors = sum(1 for gt in gts if (gt.spec.C // 8) > 1024 // nbt)  # split-K reduce launches
     stream_bytes = sum((gt.bits + 7) // 8 for gt in gts)
     value = world * n / (mean_step * 1e-3)
 
@@ -402,7 +400,7 @@ def our_arm(args):
         "clocks": clk,
         "e2e": {"value": world * n / (mean_e2e * 1e-3), "unit": "tokens/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-        "gpu_launches": args.steps * (len(gts) + nsplit_tensors),
+        "gpu_launches": args.steps * len(gts),  # one fused kernel per tensor
         "roofline": {
             "bound": "alu", "achieved": achieved_issue, "peak": issue_peak,
             "unit": "Gwarp-inst/s", "frac": achieved_issue / issue_peak,

@@ -11,7 +11,8 @@ __device__ __forceinline__ void decode_block(const LayerArgs &p, uint64_t off,
   uint32_t lo, hi;
   load_bits<RungT<S, K>::NWORDS>(p.stream, off, lo, hi);
   float I[8], scale;
-  reconstruct<S, K>(lo, hi, tab, I, scale);
+  const RungConsts<S, K> rc(p.zero);
+  reconstruct<S, K>(lo, hi, tab, rc, I, scale);
 #pragma unroll
   for (int i = 0; i < 8; ++i) Wrow[__ldg(p.perm + 8 * c + i)] = I[i] * scale;  // exact
 }

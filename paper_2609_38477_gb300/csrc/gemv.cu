@@ -1,88 +1,150 @@
-// Fused reconstruction x matrix-vector product: y = W_hat x and the decode-batch
+// Fused reconstruction x matrix-vector product: y = W_hat x, and the decode-batch
 // skinny GEMM Y = X W_hat^T (n <= 16).  W_hat is never written to memory; HBM
 // carries only the compressed stream, the plan rows and x / y.
+//
+// Work layout: a persistent kernel, one 24-warp CTA per SM.  A CTA owns a
+// contiguous range of rows (a row tile) and stages, once, the LFSR jump tables
+// and the activations in permuted column order (all columns when they fit,
+// else column chunks).  Within a tile and chunk, the row-major sequence of
+// (row, block) pairs is cut into 24 equal contiguous ranges, one per warp, so
+// every warp gets the same number of blocks whatever the row length.  Rows cut
+// by a range boundary leave per-warp partial sums in shared memory that are
+// added in warp order, so results are deterministic.
 #include <cuda_fp16.h>
 
 #include "seedq_internal.cuh"
 
 namespace seedq {
 
-constexpr int kThreads = 256;           // 8 warps
-constexpr int kWarps = kThreads / 32;
-constexpr int kXFloats = 8192;          // 32 KB of staged activations per CTA
-
-// Column blocks per split for batch n: the activation slice of a split
-// (n x 8 cb floats, permuted order) fills the 32 KB staging buffer.
-__host__ __device__ inline int cb_for(int n) { return kXFloats / 8 / n; }
-
-// Batch sizes run by one of the instantiated kernels: 1, 2, 4, 8, 16.
-__host__ __device__ inline int batch_template(int n) {
-  return n <= 1 ? 1 : n <= 2 ? 2 : n <= 4 ? 4 : n <= 8 ? 8 : 16;
-}
-
-// Split-K partial sums the layer must hold for batches up to max_batch.
-int64_t gemv_partial_elems(const seedq_layer *L, int max_batch) {
-  int64_t need = 0;
-  for (int nt = 1; nt <= batch_template(max_batch); nt *= 2) {
-    const int cb = cb_for(nt);
-    const int64_t ns = (L->args.nb + cb - 1) / cb;
-    const int64_t e = ns > 1 ? ns * (nt < max_batch ? nt : max_batch) * L->args.R : 0;
-    if (e > need) need = e;
-  }
-  return need;
-}
+constexpr int kWarps = 24;
+constexpr int kThreads = kWarps * 32;
+constexpr int kXBytes = 112 * 1024;     // staged activations per CTA
+constexpr int kAccFloats = 8192;        // row-tile accumulators per CTA (rows x n)
 
 struct GemvArgs {
   LayerArgs p;
   const uint16_t *x;  // n x C bf16, original column order
   float *y;           // n x R
-  float *partials;    // nsplit x n x R
   int n;
-  int cb;
-  int nsplit;
-  int64_t nrt;        // row tiles (kWarps rows each)
-  int64_t ntiles;
+  int cw;             // column blocks per chunk
+  int nchunks;
+  int rt;             // rows per tile
+  int ntiles;
+  uint32_t zero;      // 0 at run time; keeps per-rung constants in registers
 };
+
+__host__ __device__ inline int batch_template(int n) {
+  return n <= 1 ? 1 : n <= 2 ? 2 : n <= 4 ? 4 : n <= 8 ? 8 : 16;
+}
 
 __device__ __forceinline__ float bf16_to_f32(uint16_t b) { return __uint_as_float((uint32_t)b << 16); }
 
-// One block of rung (S,K): reconstruct exactly, then acc[b] += scale * sum_i I_i x_b,i.
 template <int S, int K, int NB>
-__device__ __forceinline__ void gemv_block(const LayerArgs &p, uint64_t off, const uint64_t *tab,
-                                           const float *xc, int xstride, float (&acc)[NB]) {
-  uint32_t lo, hi;
-  load_bits<RungT<S, K>::NWORDS>(p.stream, off, lo, hi);
+__device__ __forceinline__ void block_fma(const uint32_t (&w)[3], uint32_t sh, const uint64_t *tab,
+                                          const RungConsts<S, K> &rc, const float *xc,
+                                          int xstride, float (&acc)[NB]) {
+  const uint32_t lo = __funnelshift_r(w[0], w[1], sh);
+  const uint32_t hi = __funnelshift_r(w[1], w[2], sh);
   float I[8], scale;
-  reconstruct<S, K>(lo, hi, tab, I, scale);
+  reconstruct<S, K>(lo, hi, tab, rc, I, scale);
 #pragma unroll
   for (int b = 0; b < NB; ++b) {
     const float4 x0 = *reinterpret_cast<const float4 *>(xc + b * xstride);
     const float4 x1 = *reinterpret_cast<const float4 *>(xc + b * xstride + 4);
-    float s = I[0] * x0.x;
-    s = __fmaf_rn(I[1], x0.y, s);
-    s = __fmaf_rn(I[2], x0.z, s);
-    s = __fmaf_rn(I[3], x0.w, s);
-    s = __fmaf_rn(I[4], x1.x, s);
-    s = __fmaf_rn(I[5], x1.y, s);
-    s = __fmaf_rn(I[6], x1.z, s);
-    s = __fmaf_rn(I[7], x1.w, s);
-    acc[b] = __fmaf_rn(scale, s, acc[b]);
+    float sacc = I[0] * x0.x;
+    sacc = __fmaf_rn(I[1], x0.y, sacc);
+    sacc = __fmaf_rn(I[2], x0.z, sacc);
+    sacc = __fmaf_rn(I[3], x0.w, sacc);
+    sacc = __fmaf_rn(I[4], x1.x, sacc);
+    sacc = __fmaf_rn(I[5], x1.y, sacc);
+    sacc = __fmaf_rn(I[6], x1.z, sacc);
+    sacc = __fmaf_rn(I[7], x1.w, sacc);
+    acc[b] = __fmaf_rn(scale, sacc, acc[b]);
   }
 }
 
+// Blocks [s0, s0 + nblk) of one row, all at rung (S,K).  Lanes take
+// consecutive blocks; 32 consecutive blocks span exactly L words, so each
+// lane's in-word shift is fixed and its word pointer steps by L.  Words are
+// loaded one group ahead.  xc0 points at the staged activations of block s0.
+template <int S, int K, int NB>
+__device__ __forceinline__ void run_segment(const uint32_t *__restrict__ base, uint32_t bit0,
+                                            int nblk, const uint64_t *tab, const float *xc0,
+                                            int xstride, int lane, uint32_t z, float (&acc)[NB]) {
+  constexpr int L = RungT<S, K>::L;
+  constexpr int NW = RungT<S, K>::NWORDS;
+  const RungConsts<S, K> rc(z);
+  const uint32_t b0 = bit0 + (uint32_t)lane * L;
+  const uint32_t sh = b0 & 31;
+  const uint32_t *q = base + (b0 >> 5);
+  const float *xc = xc0 + lane * 8;
+  const int ngroups = (nblk + 31) >> 5;
+  int left = nblk - lane;  // blocks from this lane's current one to the segment end
+  uint32_t w[3] = {0u, 0u, 0u};
+  if (left > 0) {
+#pragma unroll
+    for (int i = 0; i < NW; ++i) w[i] = __ldg(q + i);
+  }
+  for (int g = 0; g < ngroups; ++g) {
+    const uint32_t cur[3] = {w[0], w[1], w[2]};
+    const bool mine = left > 0;
+    left -= 32;
+    q += L;
+    if (left > 0) {
+#pragma unroll
+      for (int i = 0; i < NW; ++i) w[i] = __ldg(q + i);
+    }
+    if (mine) block_fma<S, K, NB>(cur, sh, tab, rc, xc, xstride, acc);
+    xc += 256;
+  }
+}
+
+// Blocks [ca, cb) of row r (a column range inside the staged chunk starting at
+// block cb0).  Rungs are non-decreasing along a row, so the range crosses at
+// most J rung segments; each runs a loop specialized for its rung.  Returns
+// the warp-wide sums in acc (every lane holds them).
 template <int NB>
-__device__ __forceinline__ void dispatch_block(int code, const LayerArgs &p, uint64_t off,
-                                               const uint64_t *tab, const float *xc, int xstride,
-                                               float (&acc)[NB]) {
-  switch (code) {
-#define SEEDQ_CASE(S_, K_)                                      \
-  case rung_code(S_, K_):                                       \
-    gemv_block<S_, K_, NB>(p, off, tab, xc, xstride, acc);      \
+__device__ __forceinline__ void row_range(const GemvArgs &a, const uint64_t *tabs, const float *xs,
+                                          int64_t r, int ca, int cb, int cb0, int lane,
+                                          float (&acc)[NB]) {
+  const LayerArgs &p = a.p;
+  const int J = p.J;
+  const uint64_t roff = __ldg(p.row_off + r);
+  const uint32_t *base = p.stream + (roff >> 5);
+  const uint32_t rbit = (uint32_t)(roff & 31);
+  const int xstride = a.cw * 8;
+#pragma unroll
+  for (int b = 0; b < NB; ++b) acc[b] = 0.f;
+  uint32_t seg_bits = 0;  // bits of the row before block `lo`
+  int lo = 0;
+  for (int j = 0; j < J && lo < cb; ++j) {
+    const int hi = (j < J - 1) ? __ldg(p.brk + r * (J - 1) + j) : p.nb;
+    const int Lj = p.L[j];
+    const int s0 = max(lo, ca), s1 = min(hi, cb);
+    if (s0 < s1) {
+      const uint32_t bit0 = rbit + seg_bits + (uint32_t)(s0 - lo) * Lj;
+      const uint64_t *tab = tabs + p.slot[j] * 512;
+      const float *xc0 = xs + (s0 - cb0) * 8;
+      switch (p.code[j]) {
+#define SEEDQ_CASE(S_, K_)                                                                  \
+  case rung_code(S_, K_):                                                                   \
+    run_segment<S_, K_, NB>(base, bit0, s1 - s0, tab, xc0, xstride, lane, a.zero, acc);     \
     break;
-    SEEDQ_FOR_EACH_RUNG(SEEDQ_CASE)
+        SEEDQ_FOR_EACH_RUNG(SEEDQ_CASE)
 #undef SEEDQ_CASE
-    default:
-      break;
+        default:
+          break;
+      }
+    }
+    seg_bits += (uint32_t)(hi - lo) * Lj;
+    lo = hi;
+  }
+#pragma unroll
+  for (int b = 0; b < NB; ++b) {
+    float v = acc[b];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    acc[b] = v;
   }
 }
 
@@ -96,149 +158,134 @@ __device__ __forceinline__ float outlier_term(const GemvArgs &a, int64_t r, int 
   return s;
 }
 
-// One warp, one row, one column split [cb0, cb1): lanes take consecutive blocks.
-// Rungs are non-decreasing along a row, so almost every group of 32 blocks has a
-// single rung: then lane offsets are base + lane * l(g), and the rung dispatch
-// is warp-uniform.  Groups that straddle a breakpoint run once per rung present.
 template <int NB>
-__device__ void gemv_row(const GemvArgs &a, const uint64_t *tabs, const float *xs, int64_t r,
-                         int s, int cb0, int cb1, int lane) {
-  const LayerArgs &p = a.p;
-  const int J = p.J;
-  int32_t bk[kMaxJ];
-#pragma unroll
-  for (int j = 0; j < kMaxJ - 1; ++j) bk[j] = (j < J - 1) ? __ldg(p.brk + r * (J - 1) + j) : p.nb;
-  uint64_t off = __ldg(p.row_off + r) + bits_before(bk, J, p.L, p.nb, cb0);
-  const int xstride = a.cb * 8;
-  float acc[NB];
-#pragma unroll
-  for (int b = 0; b < NB; ++b) acc[b] = 0.f;
-  int seg = rung_of(bk, J, cb0);
-  for (int g0 = cb0; g0 < cb1; g0 += 32) {
-    const int gend = min(g0 + 32, cb1);
-    while (seg < J - 1 && bk[seg] <= g0) ++seg;
-    const int c = g0 + lane;
-    const bool valid = c < gend;
-    const float *xc = xs + (c - cb0) * 8;
-    const int seg_end = (seg < J - 1) ? bk[seg] : p.nb;
-    if (seg_end >= gend) {
-      const int Lg = p.L[seg];
-      if (valid)
-        dispatch_block<NB>(p.code[seg], p, off + (uint64_t)lane * Lg,
-                           tabs + p.slot[seg] * 512, xc, xstride, acc);
-      off += (uint64_t)(gend - g0) * Lg;
-    } else {
-      const int myr = rung_of(bk, J, c);
-      const uint64_t base = bits_before(bk, J, p.L, p.nb, g0);
-      const uint64_t myoff = off + (bits_before(bk, J, p.L, p.nb, c) - base);
-      const int last = rung_of(bk, J, gend - 1);
-      for (int rr = seg; rr <= last; ++rr)
-        if (valid && myr == rr)
-          dispatch_block<NB>(p.code[rr], p, myoff, tabs + p.slot[rr] * 512, xc, xstride, acc);
-      off += bits_before(bk, J, p.L, p.nb, gend) - base;
-    }
-  }
-#pragma unroll
-  for (int b = 0; b < NB; ++b) {
-    float v = acc[b];
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    acc[b] = v;
-  }
-  if (lane == 0) {
-    for (int b = 0; b < a.n && b < NB; ++b) {
-      if (a.nsplit == 1) a.y[(int64_t)b * p.R + r] = acc[b] + outlier_term(a, r, b);
-      else a.partials[((int64_t)s * a.n + b) * p.R + r] = acc[b];
-    }
-  }
-}
-
-template <int NB>
-__global__ void __launch_bounds__(kThreads) k_gemv(const __grid_constant__ GemvArgs a) {
+__global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ GemvArgs a) {
   extern __shared__ __align__(16) uint64_t smem[];
   const LayerArgs &p = a.p;
   uint64_t *tabs = smem;
   float *xs = reinterpret_cast<float *>(smem + p.nslots * 512);
-  for (int i = threadIdx.x; i < p.nslots * 512; i += kThreads) tabs[i] = __ldg(p.tables + i);
+  float *racc = xs + NB * a.cw * 8;               // rt x NB row accumulators
+  float *slot = racc + a.rt * NB;                 // kWarps x 2 x NB partial sums
+  int *slot_row = reinterpret_cast<int *>(slot + kWarps * 2 * NB);
+  {
+    const uint4 *src = reinterpret_cast<const uint4 *>(p.tables);
+    uint4 *dst = reinterpret_cast<uint4 *>(tabs);
+    for (int i = threadIdx.x; i < p.nslots * 256; i += kThreads) dst[i] = __ldg(src + i);
+  }
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  int cur_s = -1;
-  for (int64_t t = blockIdx.x; t < a.ntiles; t += gridDim.x) {
-    const int s = (int)(t / a.nrt);
-    const int64_t rt = t - (int64_t)s * a.nrt;
-    const int cb0 = s * a.cb, cb1 = min(cb0 + a.cb, p.nb);
-    if (s != cur_s) {
+  for (int tile = blockIdx.x; tile < a.ntiles; tile += gridDim.x) {
+    const int64_t r_lo = (int64_t)tile * a.rt;
+    const int nr = (int)min((int64_t)a.rt, p.R - r_lo);
+    for (int i = threadIdx.x; i < nr * NB; i += kThreads) racc[i] = 0.f;
+    for (int ch = 0; ch < a.nchunks; ++ch) {
+      const int cb0 = ch * a.cw, cb1 = min(cb0 + a.cw, p.nb), ncb = cb1 - cb0;
       __syncthreads();
-      const int span = a.cb * 8, ncols = (cb1 - cb0) * 8;
-      for (int idx = threadIdx.x; idx < NB * span; idx += kThreads) {
-        const int b = idx / span, pc = idx - b * span;
-        float v = 0.f;
-        if (b < a.n && pc < ncols) {
-          const int col = __ldg(p.perm + cb0 * 8 + pc);
-          bool outl = false;
-          for (int o = 0; o < p.n_out; ++o) outl |= (p.out_cols[o] == col);
-          if (!outl) v = bf16_to_f32(a.x[(int64_t)b * p.C + col]);
+      // Stage the chunk's activations in permuted order (0 at outlier columns):
+      // coalesced reads of x and of the inverse permutation, scattered into
+      // shared memory, so no load waits on another.
+      for (int col0 = threadIdx.x; col0 < p.C; col0 += 4 * kThreads) {
+        int pos[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int col = col0 + u * kThreads;
+          pos[u] = (col < p.C) ? __ldg(p.invperm + col) - cb0 * 8 : -1;
         }
-        xs[idx] = v;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int col = col0 + u * kThreads;
+          if (pos[u] >= 0 && pos[u] < ncb * 8) {
+            bool outl = false;
+            for (int o = 0; o < p.n_out; ++o) outl |= (p.out_cols[o] == col);
+            for (int b = 0; b < a.n; ++b)
+              xs[b * a.cw * 8 + pos[u]] = outl ? 0.f : bf16_to_f32(__ldg(a.x + (int64_t)b * p.C + col));
+          }
+        }
+      }
+      if (threadIdx.x < kWarps * 2) slot_row[threadIdx.x] = -1;
+      __syncthreads();
+      // This warp's equal share of the tile's (row, block) pairs in the chunk.
+      const int64_t work = (int64_t)nr * ncb;
+      const int64_t wb0 = work * warp / kWarps, wb1 = work * (warp + 1) / kWarps;
+      int64_t wb = wb0;
+      while (wb < wb1) {
+        const int rr = (int)(wb / ncb);
+        const int c0 = (int)(wb - (int64_t)rr * ncb);
+        const int c1 = (int)min((int64_t)ncb, c0 + (wb1 - wb));
+        float acc[NB];
+        row_range<NB>(a, tabs, xs, r_lo + rr, cb0 + c0, cb0 + c1, cb0, lane, acc);
+        if (lane == 0) {
+          if (c0 == 0 && c1 == ncb) {  // whole row of the chunk: sole writer
+#pragma unroll
+            for (int b = 0; b < NB; ++b) racc[rr * NB + b] += acc[b];
+          } else {
+            const int s = (wb == wb0) ? 0 : 1;
+            slot_row[warp * 2 + s] = rr;
+#pragma unroll
+            for (int b = 0; b < NB; ++b) slot[(warp * 2 + s) * NB + b] = acc[b];
+          }
+        }
+        wb += c1 - c0;
       }
       __syncthreads();
-      cur_s = s;
+      // Rows cut by range boundaries: add the partial sums in warp order.
+      for (int rr = threadIdx.x; rr < nr; rr += kThreads) {
+        for (int sidx = 0; sidx < kWarps * 2; ++sidx) {
+          if (slot_row[sidx] == rr) {
+            for (int b = 0; b < NB; ++b) racc[rr * NB + b] += slot[sidx * NB + b];
+          }
+        }
+      }
     }
-    const int64_t r = rt * kWarps + warp;
-    if (r < p.R) gemv_row<NB>(a, tabs, xs, r, s, cb0, cb1, lane);
+    __syncthreads();
+    for (int i = threadIdx.x; i < nr * a.n; i += kThreads) {
+      const int rr = i / a.n, b = i - rr * a.n;
+      const int64_t r = r_lo + rr;
+      a.y[(int64_t)b * p.R + r] = racc[rr * NB + b] + outlier_term(a, r, b);
+    }
+    __syncthreads();
   }
 }
 
-// Deterministic split-K reduction (splits summed in ascending order) + outliers.
-__global__ void k_reduce(const __grid_constant__ GemvArgs a) {
-  const int64_t total = (int64_t)a.n * a.p.R;
-  for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
-       t += (int64_t)gridDim.x * blockDim.x) {
-    const int b = (int)(t / a.p.R);
-    const int64_t r = t - (int64_t)b * a.p.R;
-    float v = 0.f;
-    for (int s = 0; s < a.nsplit; ++s) v += a.partials[((int64_t)s * a.n + b) * a.p.R + r];
-    a.y[t] = v + outlier_term(a, r, b);
-  }
+template <int NB>
+static size_t smem_bytes(int nslots, int cw, int rt) {
+  return sizeof(uint64_t) * 512 * nslots + sizeof(float) * NB * cw * 8 + sizeof(float) * rt * NB +
+         sizeof(float) * kWarps * 2 * NB + sizeof(int) * kWarps * 2;
 }
 
 template <int NB>
 static seedq_status launch(const seedq_layer *L, const uint16_t *x, int n, float *y,
                            cudaStream_t st) {
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   GemvArgs a;
   a.p = L->args;
   a.x = x;
   a.y = y;
-  a.partials = L->d_partials;
   a.n = n;
-  a.cb = cb_for(NB);
-  a.nsplit = (L->args.nb + a.cb - 1) / a.cb;
-  a.nrt = (L->args.R + kWarps - 1) / kWarps;
-  a.ntiles = a.nrt * a.nsplit;
-  if (a.nsplit > 1 && (int64_t)a.nsplit * n * L->args.R > L->partial_elems) return SEEDQ_ERR_INVALID_ARG;
-  const size_t smem = sizeof(uint64_t) * 512 * L->args.nslots + sizeof(float) * NB * a.cb * 8;
+  a.zero = 0u;
+  const int cw_max = kXBytes / (int)sizeof(float) / 8 / NB;
+  a.cw = L->args.nb < cw_max ? L->args.nb : cw_max;
+  a.nchunks = (L->args.nb + a.cw - 1) / a.cw;
+  int64_t rt = (L->args.R + sms - 1) / sms;
+  if (rt * NB > kAccFloats) rt = kAccFloats / NB;
+  a.rt = (int)rt;
+  a.ntiles = (int)((L->args.R + rt - 1) / rt);
+  const size_t smem = smem_bytes<NB>(L->args.nslots, a.cw, a.rt);
   static bool attr_set = false;
   if (!attr_set) {
     SEEDQ_CUDA(cudaFuncSetAttribute(k_gemv<NB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    (int)(sizeof(uint64_t) * 512 * kMaxJ + sizeof(float) * kXFloats)));
+                                    (int)smem_bytes<NB>(kMaxJ, cw_max, kAccFloats / NB)));
     attr_set = true;
   }
-  int dev = 0, sms = 0, occ = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  SEEDQ_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k_gemv<NB>, kThreads, smem));
-  if (occ < 1) occ = 1;
-  const int64_t want = (int64_t)sms * occ;
-  const int grid = (int)(a.ntiles < want ? a.ntiles : want);
+  const int grid = a.ntiles < sms ? a.ntiles : sms;
   k_gemv<NB><<<grid, kThreads, smem, st>>>(a);
   SEEDQ_CUDA(cudaGetLastError());
-  if (a.nsplit > 1) {
-    const int64_t total = (int64_t)n * L->args.R;
-    const int g = (int)((total + 255) / 256 < (int64_t)sms * 8 ? (total + 255) / 256 : (int64_t)sms * 8);
-    k_reduce<<<g, 256, 0, st>>>(a);
-    SEEDQ_CUDA(cudaGetLastError());
-  }
   return SEEDQ_OK;
 }
+
+// The fused kernel keeps no global scratch (partial sums live in shared memory).
+int64_t gemv_partial_elems(const seedq_layer *, int) { return 0; }
 
 }  // namespace seedq
 
@@ -251,11 +298,13 @@ seedq_status seedq_gemm_small_batch(const seedq_layer *L, const uint16_t *X, int
   if (!L || !X || !Y || n < 1 || n > L->max_batch) return SEEDQ_ERR_INVALID_ARG;
   if (!L->args.stream) return SEEDQ_ERR_STREAM;
   cudaStream_t st = (cudaStream_t)cuda_stream;
-  if (n == 1) return launch<1>(L, X, n, Y, st);
-  if (n == 2) return launch<2>(L, X, n, Y, st);
-  if (n <= 4) return launch<4>(L, X, n, Y, st);
-  if (n <= 8) return launch<8>(L, X, n, Y, st);
-  return launch<16>(L, X, n, Y, st);
+  switch (batch_template(n)) {
+    case 1: return launch<1>(L, X, n, Y, st);
+    case 2: return launch<2>(L, X, n, Y, st);
+    case 4: return launch<4>(L, X, n, Y, st);
+    case 8: return launch<8>(L, X, n, Y, st);
+    default: return launch<16>(L, X, n, Y, st);
+  }
 }
 
 seedq_status seedq_gemv(const seedq_layer *L, const uint16_t *x, float *y, void *cuda_stream) {

@@ -56,6 +56,11 @@ __global__ void k_perm(const float *__restrict__ a, int C, int32_t *__restrict__
   if (i < C) perm[rank] = i;
 }
 
+__global__ void k_invperm(const int32_t *__restrict__ perm, int C, int32_t *__restrict__ inv) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < C) inv[perm[i]] = i;
+}
+
 // Block means of the permuted a, summed in channel order, and their unit-mean
 // normalization summed in ascending block order (Eq. imp; App. A.7 fixed order).
 __global__ void k_abar(const float *__restrict__ a, const int32_t *__restrict__ perm,
@@ -262,6 +267,7 @@ __global__ void k_synth(const __grid_constant__ LayerArgs p, const int32_t *__re
 static void free_layer(seedq_layer *L) {
   if (!L) return;
   cudaFree(L->d_perm);
+  cudaFree(L->d_invperm);
   cudaFree(L->d_abar);
   cudaFree(L->d_rho);
   cudaFree(L->d_rho_in);
@@ -273,6 +279,7 @@ static void free_layer(seedq_layer *L) {
   cudaFree(L->d_flags);
   cudaFree(L->d_summary);
   cudaFree(L->d_partials);
+
   free(L);
 }
 
@@ -389,6 +396,7 @@ seedq_status seedq_layer_prepare(const seedq_layer_desc *d, const seedq_schedule
     }                                                                  \
   } while (0)
   ALLOC(L->d_perm, sizeof(int32_t) * C);
+  ALLOC(L->d_invperm, sizeof(int32_t) * C);
   ALLOC(L->d_abar, sizeof(double) * nb);
   ALLOC(L->d_rho, sizeof(double) * R);
   ALLOC(L->d_a_in, sizeof(float) * C);
@@ -414,12 +422,15 @@ seedq_status seedq_layer_prepare(const seedq_layer_desc *d, const seedq_schedule
   }
   L->partial_elems = gemv_partial_elems(L, mb);
   if (L->partial_elems) ALLOC(L->d_partials, sizeof(float) * L->partial_elems);
+
 #undef ALLOC
   L->args.perm = L->d_perm;
+  L->args.invperm = L->d_invperm;
   L->args.brk = L->d_brk;
   L->args.row_off = L->d_row_off;
   L->args.tables = L->d_tables;
   L->args.flags = L->d_flags;
+
   L->args.stream = nullptr;
 
   int *dL = nullptr;
@@ -431,6 +442,7 @@ seedq_status seedq_layer_prepare(const seedq_layer_desc *d, const seedq_schedule
     e = cudaMemcpyAsync(L->d_rho_in, d->rho, sizeof(float) * R, cudaMemcpyHostToDevice, st);
   if (e == cudaSuccess) {
     k_perm<<<(int)((C + 255) / 256), 256, 0, st>>>(L->d_a_in, (int)C, L->d_perm);
+    k_invperm<<<(int)((C + 255) / 256), 256, 0, st>>>(L->d_perm, (int)C, L->d_invperm);
     k_abar<<<1, 1024, 0, st>>>(L->d_a_in, L->d_perm, nb, L->d_abar);
     k_rho<<<1, 1024, 0, st>>>(L->d_rho_in, R, L->d_rho);
     SchedArgs sa;

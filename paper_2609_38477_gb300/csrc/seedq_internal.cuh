@@ -34,7 +34,8 @@ struct LayerArgs {
   const uint64_t *row_off;  // R + 1 bit offsets
   const int32_t *brk;       // R x (J-1): first block of row r with rung > j
   const uint64_t *tables;   // nslots x 512 LFSR jump tables
-  const int32_t *perm;      // C
+  const int32_t *perm;      // C: block c holds columns perm[8c..8c+7]
+  const int32_t *invperm;   // C: position of column j in the permuted order
   const uint16_t *out_vals; // R x n_out binary16
   uint32_t *flags;
   int64_t R, C;
@@ -46,6 +47,7 @@ struct LayerArgs {
   int32_t nslots;
   int32_t n_out;
   int32_t out_cols[kMaxOutliers];
+  uint32_t zero;            // 0; see RungConsts
 };
 
 }  // namespace seedq
@@ -63,6 +65,7 @@ struct seedq_layer {
   int device;
   // owned device memory
   int32_t *d_perm;
+  int32_t *d_invperm;
   double *d_abar, *d_rho;
   float *d_rho_in, *d_a_in;
   int32_t *d_brk;
@@ -131,48 +134,159 @@ struct RungT {
   static constexpr int NWORDS = (31 + L > 64) ? 3 : 2;
 };
 
+// ---------------------------------------------------------- reconstruction
+//
 // Eq. codec for one block, exactly: I[i] = sum_j t_j (x_{iK+j} - 2^{S-1}) as an
 // fp32 integer and scale = 2^(E-S+1), so w_i = I[i] * scale (exact, |I| < 2^21).
 //
-// The LFSR sequence prefix Q (64 bits: o_0..o_63) comes from two GF(2)-linear
-// jump tables indexed by the seed's bytes (tab[v] = Q(v), tab[256+v] = Q(v<<8)).
-// Each state x_n = bits [n, n+S) of Q is turned into the float 2^S + x_n by
-// placing it under a fixed exponent; an FMA chain started at -1.5 * 2^S * sum t
-// then yields I exactly, since every partial sum is an integer below 2^24.
-template <int S, int K>
-__device__ __forceinline__ void reconstruct(uint32_t lo, uint32_t hi,
-                                            const uint64_t *tab, float (&I)[8],
-                                            float &scale) {
-  const uint64_t F = ((uint64_t)hi << 32) | lo;
-  const uint32_t seed = lo & ((1u << S) - 1u);
-  uint64_t Q = tab[seed & 255u];
-  if (S > 8) Q ^= tab[256 + (seed >> 8)];
-  const int E = ((int)(lo << (28 - S))) >> 28;  // 4-bit two's complement at bit S
-  scale = __int_as_float((127 + E - S + 1) << 23);
-  float tf[K];
-  float T = 0.f;
-#pragma unroll
+// LFSR: the 64-bit sequence prefix Q = o_0..o_63 comes from two GF(2)-linear
+// jump tables indexed by the seed's bytes: tab[v] = Q(v), tab[256+v] =
+// Q((v mod 2^(S-8)) << 8), so the raw second byte of the field word indexes it.
+//
+// States as floats: a state x_n sits at bits [n, n+S) of Q.  One funnel shift
+// brings a window of Q such that x_n lies at mantissa bits [23-S-d, 23-d) of a
+// 32-bit word; masking it and OR-ing exponent 127+S+d gives the float
+// 2^(S+d) + x_n.  A group of G consecutive states of one weight shares one
+// window (d = 0..G-1).  An FMA chain from init = -sum_j t_j (2^(S+d_j) + 2^(S-1))
+// then yields I exactly, provided every partial sum stays an integer below
+// 2^24 in magnitude; group_size() picks the largest G for which the worst case
+// (all |t_j| = 8) satisfies that.
+
+__host__ __device__ constexpr long long exact_bound(int S, int K, int G) {
+  long long s = 0;
   for (int j = 0; j < K; ++j) {
-    const int tj = ((int)((uint32_t)(F >> (S + 4 + 4 * j)) << 28)) >> 28;
-    tf[j] = (float)tj;
-    T += tf[j];
+    const int d = (K - 1 - j) % G;
+    s += 8ll * ((1ll << (S + d)) + (1ll << (S - 1)));
   }
-  const float init = (-1.5f * (float)(1 << S)) * T;
-  constexpr uint32_t EXP = (uint32_t)(127 + S) << 23;
-  constexpr uint32_t MSK = ((1u << S) - 1u) << (23 - S);
-  const uint32_t Qlo = (uint32_t)Q;
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    float acc = init;
+  return s + 48ll * (1ll << (S - 1));
+}
+
+__host__ __device__ constexpr int group_size(int S, int K) {
+  int g = 1;
+  for (int G = 1; G <= K; ++G)
+    if (exact_bound(S, K, G) < (1ll << 24) && S + G <= 24) g = G;
+  return g;
+}
+
+// Window (lo, mid, hi hold bits [0,32), [16,48), [32,64) of the block's field
+// word) and in-window bit position of the signed 4-bit field at absolute bit P;
+// the field must lie in mantissa bits [0, 23) of its window.
+__host__ __device__ constexpr int field_window(int P) { return P + 4 <= 23 ? 0 : P - 16 + 4 <= 23 ? 1 : 2; }
+__host__ __device__ constexpr int field_pos(int P) { return P - 16 * field_window(P); }
+
+// Per-rung constants kept in registers.  They are built from a runtime zero so
+// the compiler cannot fold them into instruction immediates: a LOP3 takes one
+// immediate at most, and (w & mask) | exponent must stay a single LOP3.
+template <int S, int K>
+struct RungConsts {
+  static constexpr int G = group_size(S, K);
+  uint32_t e_msk, e_x;           // shared exponent field
+  uint32_t t_msk[K], t_x[K];     // mantissa fields t_j
+  uint32_t s_msk[G], s_exp[G];   // state windows, by offset d within a group
+  __device__ __forceinline__ explicit RungConsts(uint32_t z) {
+    e_msk = (15u << S) ^ z;
+    e_x = (8u << S) ^ z;
 #pragma unroll
     for (int j = 0; j < K; ++j) {
-      const int n = i * K + j;
-      const int sh = n + S - 23;
-      const uint32_t w = (sh >= 0) ? (uint32_t)(Q >> (sh & 63)) : (Qlo << ((-sh) & 31));
-      acc = __fmaf_rn(tf[j], __int_as_float((w & MSK) | EXP), acc);
+      const int P = field_pos(S + 4 + 4 * j);
+      t_msk[j] = (15u << P) ^ z;
+      t_x[j] = ((8u << P) | ((uint32_t)(150 - P) << 23)) ^ z;
     }
-    I[i] = acc;
+#pragma unroll
+    for (int d = 0; d < G; ++d) {
+      s_msk[d] = (((1u << S) - 1u) << (23 - S - d)) ^ z;
+      s_exp[d] = ((uint32_t)(127 + S + d) << 23) ^ z;
+    }
   }
+};
+
+// Single three-input logic instructions (the compiler otherwise splits them).
+__device__ __forceinline__ uint32_t lop_and_xor(uint32_t a, uint32_t m, uint32_t x) {
+  uint32_t r;
+  asm("lop3.b32 %0, %1, %2, %3, 0x6A;" : "=r"(r) : "r"(a), "r"(m), "r"(x));  // (a & m) ^ x
+  return r;
+}
+__device__ __forceinline__ uint32_t lop_and_or(uint32_t a, uint32_t m, uint32_t x) {
+  uint32_t r;
+  asm("lop3.b32 %0, %1, %2, %3, 0xEA;" : "=r"(r) : "r"(a), "r"(m), "r"(x));  // (a & m) | x
+  return r;
+}
+
+template <int S, int K, int J = 0>
+__device__ __forceinline__ void coeffs(uint32_t lo, uint32_t mid, uint32_t hi,
+                                       const RungConsts<S, K> &rc, float (&tf)[K]) {
+  if constexpr (J < K) {
+    constexpr int P = S + 4 + 4 * J;
+    constexpr int W = field_window(P);
+    constexpr int PP = field_pos(P);
+    static_assert(PP >= 0 && PP + 4 <= 23, "field outside the mantissa");
+    const uint32_t w = (W == 0) ? lo : (W == 1) ? mid : hi;
+    // Under exponent 150-PP the field reads as 2^(23-PP) + (t ^ 8) = 2^(23-PP) + 8 + t.
+    tf[J] = __uint_as_float(lop_and_xor(w, rc.t_msk[J], rc.t_x[J])) - (float)((1 << (23 - PP)) + 8);
+    coeffs<S, K, J + 1>(lo, mid, hi, rc, tf);
+  }
+}
+
+// 32 bits of Q (qlo | qhi << 32) starting at bit SH (SH may be negative: the
+// window then begins below bit 0 and its low bits are zero).
+template <int SH>
+__device__ __forceinline__ uint32_t qwin(uint32_t qlo, uint32_t qhi) {
+  if constexpr (SH <= -32) return 0u;
+  else if constexpr (SH < 0) return qlo << (-SH);
+  else if constexpr (SH == 0) return qlo;
+  else if constexpr (SH < 32) return __funnelshift_r(qlo, qhi, SH);
+  else if constexpr (SH == 32) return qhi;
+  else return qhi >> (SH - 32);
+}
+
+template <int S, int K, int G, int I, int J>
+__device__ __forceinline__ float state_chain(uint32_t qlo, uint32_t qhi, const RungConsts<S, K> &rc,
+                                             const float (&tf)[K], float acc) {
+  if constexpr (J < 0) {
+    return acc;
+  } else {
+    // Group holding state J of weight I: its top state jt sits at d = 0.
+    constexpr int grp = (K - 1 - J) / G;
+    constexpr int jt = K - 1 - grp * G;
+    constexpr int d = jt - J;
+    const uint32_t win = qwin<I * K + jt + S - 23>(qlo, qhi);
+    acc = __fmaf_rn(tf[J], __uint_as_float(lop_and_or(win, rc.s_msk[d], rc.s_exp[d])), acc);
+    return state_chain<S, K, G, I, J - 1>(qlo, qhi, rc, tf, acc);
+  }
+}
+
+template <int S, int K, int G, int I>
+__device__ __forceinline__ void weights_from(uint32_t qlo, uint32_t qhi, const RungConsts<S, K> &rc,
+                                             const float (&tf)[K], float init, float (&Iv)[8]) {
+  if constexpr (I < 8) {
+    Iv[I] = state_chain<S, K, G, I, K - 1>(qlo, qhi, rc, tf, init);
+    weights_from<S, K, G, I + 1>(qlo, qhi, rc, tf, init, Iv);
+  }
+}
+
+// lo, hi: the block's 64 field bits starting at its first bit.
+template <int S, int K>
+__device__ __forceinline__ void reconstruct(uint32_t lo, uint32_t hi, const uint64_t *tab,
+                                            const RungConsts<S, K> &rc, float (&I)[8],
+                                            float &scale) {
+  constexpr int G = RungConsts<S, K>::G;
+  static_assert(exact_bound(S, K, G) < (1ll << 24), "FMA chain would round");
+  uint64_t Q = tab[lo & 255u];
+  if (S > 8) Q ^= tab[256 + __byte_perm(lo, 0, 0x4441)];
+  const uint32_t qlo = (uint32_t)Q, qhi = (uint32_t)(Q >> 32);
+  // scale = 2^(E-S+1): (E+8) = field ^ 8 lands in the exponent via one multiply-add.
+  const uint32_t e8 = lop_and_xor(lo, rc.e_msk, rc.e_x);
+  scale = __uint_as_float(e8 * (1u << (23 - S)) + ((uint32_t)(127 - S + 1 - 8) << 23));
+  const uint32_t mid = __funnelshift_r(lo, hi, 16);
+  float tf[K];
+  coeffs<S, K>(lo, mid, hi, rc, tf);
+  float init = 0.f;
+#pragma unroll
+  for (int j = 0; j < K; ++j) {
+    const int d = (K - 1 - j) % G;
+    init = __fmaf_rn(tf[j], -(float)((1 << (S + d)) + (1 << (S - 1))), init);
+  }
+  weights_from<S, K, G, 0>(qlo, qhi, rc, tf, init, I);
 }
 
 __host__ __device__ inline uint64_t stream_bytes_required(uint64_t bits) {
