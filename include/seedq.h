@@ -185,6 +185,33 @@ seedq_status seedq_synth_stream(const seedq_layer *layer, uint64_t key,
                                 void *stream, uint64_t stream_bytes,
                                 void *cuda_stream);
 
+/* Allocation-free per-row schedule pass, for callers that cannot call
+ * cudaMalloc when they need it (a fixed memory budget reserved up front, an
+ * allocator-less runtime, code that must not touch the CUDA allocator while
+ * other work is in flight).  The paper has no counterpart: it is the row part
+ * of seedq_layer_prepare (Eq. ladder breakpoints, the tie pass, row bit
+ * offsets) run on caller buffers, with its temporary per-row tie counts in a
+ * file-scope device array of SEEDQ_STATIC_PLAN_MAX_ROWS entries (512 KiB held
+ * by every GPU that loads the library until exit).  It allocates nothing.
+ *   abar      device, nb doubles: unit-mean block means of the permuted a.
+ *   rho       device, rows doubles: unit-mean row factors (all 1 if none).
+ *   rows, nb  R (1..SEEDQ_STATIC_PLAN_MAX_ROWS) and C/8; larger R returns
+ *             SEEDQ_ERR_UNSUPPORTED.
+ *   brk       device, rows x (J-1) int32 out: first block of each row with
+ *             rung > j (may be NULL when J == 1).
+ *   row_off   device, rows + 1 uint64 out (row_off[rows] = total bits).
+ *   summary   device, 2 uint64 out: tied blocks at theta[j_tie], total bits;
+ *             the caller checks tie_count <= summary[0].
+ * The first call on a device looks up the array's device address with that
+ * device current, so make it before any stream capture.  Work is enqueued on
+ * cuda_stream and not waited for.  Calls share the array: calls that overlap
+ * on the GPU (other streams, other threads) race and must be serialized. */
+#define SEEDQ_STATIC_PLAN_MAX_ROWS (1 << 17)
+seedq_status seedq_row_plan_static(const double *abar, const double *rho, int64_t rows,
+                                   int32_t nb, const seedq_schedule *sched,
+                                   int64_t tie_count, int32_t *brk, uint64_t *row_off,
+                                   uint64_t *summary, void *cuda_stream);
+
 const char *seedq_status_string(seedq_status status);
 const char *seedq_last_cuda_error_string(void);
 

@@ -575,3 +575,90 @@ seedq_status seedq_synth_stream(const seedq_layer *L, uint64_t key, void *stream
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Allocation-free row pass.  Some callers cannot call cudaMalloc at the moment
+// they need a plan: code running inside a fixed memory budget reserved up
+// front, allocator-less embedded runtimes, or code that must not touch the
+// CUDA allocator while other work is in flight.  For them the per-row part of
+// the plan (ladder breakpoints, tie pass, row offsets) can run with its
+// temporary per-row tie counts kept in this file-scope device array instead of
+// layer-owned memory.  Every GPU that loads the library holds the array until
+// the process exits.  All calls share it, so calls that overlap on the GPU race.
+namespace seedq {
+
+constexpr int64_t kStaticPlanMaxRows = 1 << 17;
+
+struct StaticPlanScratch {
+  int32_t tcnt[kStaticPlanMaxRows];
+  int32_t L[kMaxJ];
+};
+
+static __device__ __align__(256) StaticPlanScratch g_static_plan_scratch;
+
+// Device address of the array, looked up once per device with that device
+// current (in host code the symbol is only a host-side stand-in).
+static StaticPlanScratch *static_scratch_ptr(seedq_status *st) {
+  static StaticPlanScratch *ptrs[64] = {nullptr};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess || dev < 0 || dev >= 64) {
+    *st = e != cudaSuccess ? cuda_fail(e) : SEEDQ_ERR_UNSUPPORTED;
+    return nullptr;
+  }
+  if (!ptrs[dev]) {
+    void *p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_static_plan_scratch);
+    if (e != cudaSuccess) {
+      *st = cuda_fail(e);
+      return nullptr;
+    }
+    ptrs[dev] = (StaticPlanScratch *)p;
+  }
+  *st = SEEDQ_OK;
+  return ptrs[dev];
+}
+
+}  // namespace seedq
+
+extern "C" seedq_status seedq_row_plan_static(const double *abar, const double *rho, int64_t rows,
+                                              int32_t nb, const seedq_schedule *s,
+                                              int64_t tie_count, int32_t *brk, uint64_t *row_off,
+                                              uint64_t *summary, void *cuda_stream) {
+  if (!abar || !rho || !s || !row_off || !summary || rows < 1 || nb < 1) return SEEDQ_ERR_INVALID_ARG;
+  if (rows > kStaticPlanMaxRows) return SEEDQ_ERR_UNSUPPORTED;
+  if (nb > kMaxCols / 8) return SEEDQ_ERR_UNSUPPORTED;
+  if (s->J < 1 || s->J > kMaxJ || !s->rungs || (s->J > 1 && (!s->theta || !brk)))
+    return SEEDQ_ERR_SCHEDULE;
+  for (int j = 0; j < s->J; ++j) {
+    if (!rung_supported(s->rungs[j].S, s->rungs[j].k)) return SEEDQ_ERR_UNSUPPORTED;
+    if (j > 0 && s->rungs[j].S + 4 * s->rungs[j].k <= s->rungs[j - 1].S + 4 * s->rungs[j - 1].k)
+      return SEEDQ_ERR_SCHEDULE;
+  }
+  for (int j = 0; j + 1 < s->J; ++j) {
+    if (!isfinite(s->theta[j])) return SEEDQ_ERR_SCHEDULE;
+    if (j > 0 && !(s->theta[j] > s->theta[j - 1])) return SEEDQ_ERR_SCHEDULE;
+  }
+  if (s->j_tie < -1 || s->j_tie >= s->J - 1 || !isfinite(s->q) || tie_count < 0) return SEEDQ_ERR_SCHEDULE;
+  if (s->j_tie < 0 && tie_count != 0) return SEEDQ_ERR_SCHEDULE;
+  seedq_status st = SEEDQ_OK;
+  StaticPlanScratch *scr = static_scratch_ptr(&st);
+  if (!scr) return st;
+  cudaStream_t cs = (cudaStream_t)cuda_stream;
+  int32_t L[kMaxJ] = {0};
+  for (int j = 0; j < s->J; ++j) L[j] = s->rungs[j].S + 4 * s->rungs[j].k + 4;
+  SEEDQ_CUDA(cudaMemcpyAsync(scr->L, L, sizeof L, cudaMemcpyHostToDevice, cs));
+  SchedArgs sa;
+  sa.J = s->J;
+  sa.j_tie = s->j_tie;
+  sa.q = s->q;
+  for (int j = 0; j < kMaxJ; ++j) sa.theta[j] = (j + 1 < s->J) ? s->theta[j] : 0.0;
+  // k_rows writes every row's tie count before k_scan reads it, so the shared
+  // array needs no clearing; with a single rung there are no ties to count.
+  if (s->J > 1)
+    k_rows<<<(int)((rows + 255) / 256), 256, 0, cs>>>(abar, rho, nb, rows, sa, brk, scr->tcnt);
+  k_scan<<<1, 1024, 0, cs>>>(rows, s->J, nb, s->J > 1 ? s->j_tie : -1, tie_count, scr->L, brk,
+                             scr->tcnt, row_off, summary);
+  SEEDQ_CUDA(cudaGetLastError());
+  return SEEDQ_OK;
+}

@@ -66,6 +66,9 @@ SIGNATURES = {
     "seedq_last_device_error": (C.c_int, [C.c_void_p, C.POINTER(C.c_uint32)]),
     "seedq_lfsr_taps": (C.c_uint32, [C.c_int32]),
     "seedq_synth_stream": (C.c_int, [C.c_void_p, C.c_uint64, C.c_void_p, C.c_uint64, C.c_void_p]),
+    "seedq_row_plan_static": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int64, C.c_int32,
+                                        C.POINTER(Schedule), C.c_int64, C.c_void_p, C.c_void_p,
+                                        C.c_void_p, C.c_void_p]),
     "seedq_status_string": (C.c_char_p, [C.c_int]),
     "seedq_last_cuda_error_string": (C.c_char_p, []),
 }
@@ -208,3 +211,17 @@ class Layer:
         f = C.c_uint32()
         _check(lib().seedq_last_device_error(self.h, C.byref(f)), "seedq_last_device_error")
         return f.value
+
+
+STATIC_PLAN_MAX_ROWS = 1 << 17
+
+
+def row_plan_static(abar, rho, rows: int, nb: int, rungs, theta, j_tie: int, q: float,
+                    tie_count: int, brk, row_off, summary, stream=None):
+    """seedq_row_plan_static: the allocation-free row pass (device buffers in/out)."""
+    rr = (Rung * len(rungs))(*[Rung(int(S), int(k)) for S, k in rungs])
+    th = np.ascontiguousarray(theta if len(theta) else [0.0], np.float64)
+    sched = Schedule(len(rungs), rr, th.ctypes.data_as(C.POINTER(C.c_double)), int(j_tie), float(q))
+    _check(lib().seedq_row_plan_static(_ptr(abar), _ptr(rho), rows, nb, C.byref(sched), tie_count,
+                                       _ptr(brk), _ptr(row_off), _ptr(summary), _stream(stream)),
+           "seedq_row_plan_static")
