@@ -154,6 +154,16 @@ seedq_status seedq_gemv(const seedq_layer *layer, const uint16_t *x, float *y,
 seedq_status seedq_gemm_small_batch(const seedq_layer *layer, const uint16_t *X,
                                     int32_t n, float *Y, void *cuda_stream);
 
+/* Several tensors in one launch (Alg. 2: tensors are decoded "in any order",
+ * so the tensors of a decode step are independent): for i < count,
+ * Y[i] = X[i] W_hat_i^T with X[i] device n x C_i bfloat16 and Y[i] device
+ * n x R_i float32, as seedq_gemm_small_batch does for one layer.  count is
+ * 1..8 and every layer must be bound and allow batch n.  Work is split across
+ * the SMs by the modeled cost of all tensors together. */
+seedq_status seedq_gemm_multi(const seedq_layer *const *layers, int32_t count,
+                              const uint16_t *const *X, int32_t n, float *const *Y,
+                              void *cuda_stream);
+
 /* Host copy of the rung index (0..J-1) of blocks of rows [row0, row0+nrows):
  * rungs_host receives nrows x (C/8) bytes.  Synchronous. */
 seedq_status seedq_layer_rung_map(const seedq_layer *layer, int64_t row0,

@@ -1,36 +1,68 @@
 // Fused reconstruction x matrix-vector product: y = W_hat x, and the decode-batch
-// skinny GEMM Y = X W_hat^T (n <= 16).  W_hat is never written to memory; HBM
-// carries only the compressed stream, the plan rows and x / y.
+// skinny GEMM Y = X W_hat^T (n <= 16), for one tensor or for several tensors
+// in one launch (the tensors of a decode step are independent: Alg. 2 decodes
+// them "in any order").  W_hat is never written to memory; HBM carries only
+// the compressed streams, the plan rows and x / y.
 //
-// Work layout: a persistent kernel, one 24-warp CTA per SM.  A CTA owns a
-// contiguous range of rows (a row tile) and stages, once, the LFSR jump tables
-// and the activations in permuted column order (all columns when they fit,
-// else column chunks).  Within a tile and chunk, the row-major sequence of
-// (row, block) pairs is cut into 24 equal contiguous ranges, one per warp, so
-// every warp gets the same number of blocks whatever the row length.  Rows cut
-// by a range boundary leave per-warp partial sums in shared memory that are
-// added in warp order, so results are deterministic.
+// Layout: a lane owns a row.  A warp takes 32 rows (a row group, in the plan's
+// row order, which puts rows with equal or nearby rung breakpoints together)
+// and walks their blocks column by column, so all lanes usually sit at the
+// same rung: control flow is uniform and the activations of a column are one
+// broadcast read.  A warp stages the stream bytes of its 32 rows, a few
+// columns at a time, into shared memory with cp.async (double-buffered),
+// together with the column slice of the activations (permuted once per call
+// into scratch by a small pre-kernel).
+//
+// Work split: all (tensor, row group, block) units in one sequence, cut into
+// one contiguous range per CTA (one CTA per SM) of equal modeled cost.  A CTA
+// processes its range in rounds of a few row groups of one tensor; the round's
+// stages are dealt round-robin to its 12 warps, whose partial sums are added
+// in warp order in shared memory.  A row group cut by a CTA boundary leaves
+// one partial sum per CTA in scratch; the CTA that arrives last adds them in
+// CTA order.  No result depends on timing.
 #include <cuda_fp16.h>
 
 #include "seedq_internal.cuh"
 
 namespace seedq {
 
-constexpr int kWarps = 24;
+constexpr int kWarps = 12;
 constexpr int kThreads = kWarps * 32;
-constexpr int kXBytes = 112 * 1024;     // staged activations per CTA
-constexpr int kAccFloats = 8192;        // row-tile accumulators per CTA (rows x n)
+constexpr int kMaxTensors = 8;
+constexpr int kMaxCtas = 256;
 
-struct GemvArgs {
+template <int NB>
+struct Cfg {
+  // Columns per stage and row groups per round, sized so 12 warps' double
+  // buffers and the round's partial sums fit in shared memory.
+  static constexpr int ST = NB == 1 ? 24 : NB == 2 ? 16 : NB <= 8 ? 8 : 4;
+  static constexpr int RG = NB <= 4 ? 4 : 1;
+  // 16-byte pieces per staged row: ST blocks of at most 44 bits, the 96-bit
+  // read-ahead of the last block, and up to 15 + 15 bytes of alignment.
+  static constexpr int PIECES = (ST * 44 / 8 + 12 + 30 + 15) / 16 + 1;
+  // Row stride in words: 16-byte aligned with an odd number of 16-byte pieces,
+  // so 8 consecutive rows start in 8 different bank groups.
+  static constexpr int RW = (PIECES % 2) ? PIECES * 4 : PIECES * 4 + 4;
+  static constexpr int STREAM_WORDS = 2 * 32 * RW;  // per warp, double-buffered
+  static constexpr int XFLOATS = 2 * ST * 8 * NB;   // per warp, double-buffered
+  static constexpr int WARP_BYTES = STREAM_WORDS * 4 + XFLOATS * 4 + 2 * 32 * 8 * 4;
+};
+
+struct TensorArgs {
   LayerArgs p;
-  const uint16_t *x;  // n x C bf16, original column order
-  float *y;           // n x R
+  const uint16_t *x;      // n x C bf16, original column order
+  float *y;               // n x R
+  int64_t ubegin;         // first unit of this tensor in the launch's sequence
+  uint64_t stream_bytes;  // readable bytes of the bound stream buffer
+};
+
+struct MultiArgs {
+  TensorArgs t[kMaxTensors];
+  int nt;
   int n;
-  int cw;             // column blocks per chunk
-  int nchunks;
-  int rt;             // rows per tile
-  int ntiles;
-  uint32_t zero;      // 0 at run time; keeps per-rung constants in registers
+  int ctas;
+  uint32_t zero;  // 0 at run time; keeps per-rung constants in registers
+  int64_t cta_begin[kMaxCtas + 1];
 };
 
 __host__ __device__ inline int batch_template(int n) {
@@ -38,6 +70,25 @@ __host__ __device__ inline int batch_template(int n) {
 }
 
 __device__ __forceinline__ float bf16_to_f32(uint16_t b) { return __uint_as_float((uint32_t)b << 16); }
+
+__device__ __forceinline__ void cp_async16(void *smem_dst, const void *gsrc) {
+  const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d), "l"(gsrc) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+// CTA whose range holds unit u.
+__device__ __forceinline__ int cta_of(const MultiArgs &a, int64_t u) {
+  int lo = 0, hi = a.ctas - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (a.cta_begin[mid] <= u) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
 
 template <int S, int K, int NB>
 __device__ __forceinline__ void block_fma(const uint32_t (&w)[3], uint32_t sh, const uint64_t *tab,
@@ -51,241 +102,453 @@ __device__ __forceinline__ void block_fma(const uint32_t (&w)[3], uint32_t sh, c
   for (int b = 0; b < NB; ++b) {
     const float4 x0 = *reinterpret_cast<const float4 *>(xc + b * xstride);
     const float4 x1 = *reinterpret_cast<const float4 *>(xc + b * xstride + 4);
-    float sacc = I[0] * x0.x;
-    sacc = __fmaf_rn(I[1], x0.y, sacc);
-    sacc = __fmaf_rn(I[2], x0.z, sacc);
-    sacc = __fmaf_rn(I[3], x0.w, sacc);
-    sacc = __fmaf_rn(I[4], x1.x, sacc);
-    sacc = __fmaf_rn(I[5], x1.y, sacc);
-    sacc = __fmaf_rn(I[6], x1.z, sacc);
-    sacc = __fmaf_rn(I[7], x1.w, sacc);
-    acc[b] = __fmaf_rn(scale, sacc, acc[b]);
+    float s0 = I[0] * x0.x, s1 = I[4] * x1.x;
+    s0 = __fmaf_rn(I[1], x0.y, s0);
+    s1 = __fmaf_rn(I[5], x1.y, s1);
+    s0 = __fmaf_rn(I[2], x0.z, s0);
+    s1 = __fmaf_rn(I[6], x1.z, s1);
+    s0 = __fmaf_rn(I[3], x0.w, s0);
+    s1 = __fmaf_rn(I[7], x1.w, s1);
+    acc[b] = __fmaf_rn(scale, s0 + s1, acc[b]);
   }
 }
 
-// Blocks [s0, s0 + nblk) of one row, all at rung (S,K).  Lanes take
-// consecutive blocks; 32 consecutive blocks span exactly L words, so each
-// lane's in-word shift is fixed and its word pointer steps by L.  Words are
-// loaded one group ahead.  xc0 points at the staged activations of block s0.
+// n consecutive columns of this lane's row at rung (S,K): pos is the bit
+// position of the first block in the lane's staged row buffer (advanced by
+// n * l(g)); xc the staged activations of the first column.
 template <int S, int K, int NB>
-__device__ __forceinline__ void run_segment(const uint32_t *__restrict__ base, uint32_t bit0,
-                                            int nblk, const uint64_t *tab, const float *xc0,
-                                            int xstride, int lane, uint32_t z, float (&acc)[NB]) {
+__device__ __forceinline__ void run_cols(const uint32_t *rowbuf, uint32_t &pos, int n,
+                                         const uint64_t *tab, const float *xc, int xstride,
+                                         uint32_t z, float (&acc)[NB]) {
   constexpr int L = RungT<S, K>::L;
-  constexpr int NW = RungT<S, K>::NWORDS;
   const RungConsts<S, K> rc(z);
-  const uint32_t b0 = bit0 + (uint32_t)lane * L;
-  const uint32_t sh = b0 & 31;
-  const uint32_t *q = base + (b0 >> 5);
-  const float *xc = xc0 + lane * 8;
-  const int ngroups = (nblk + 31) >> 5;
-  int left = nblk - lane;  // blocks from this lane's current one to the segment end
-  uint32_t w[3] = {0u, 0u, 0u};
-  if (left > 0) {
-#pragma unroll
-    for (int i = 0; i < NW; ++i) w[i] = __ldg(q + i);
+  uint32_t w[3];
+  {
+    const uint32_t *q = rowbuf + (pos >> 5);
+    w[0] = q[0];
+    w[1] = q[1];
+    w[2] = q[2];
   }
-  for (int g = 0; g < ngroups; ++g) {
+  for (int i = 0; i < n; ++i) {
     const uint32_t cur[3] = {w[0], w[1], w[2]};
-    const bool mine = left > 0;
-    left -= 32;
-    q += L;
-    if (left > 0) {
-#pragma unroll
-      for (int i = 0; i < NW; ++i) w[i] = __ldg(q + i);
+    const uint32_t sh = pos & 31;
+    pos += L;
+    if (i + 1 < n) {
+      const uint32_t *q = rowbuf + (pos >> 5);
+      w[0] = q[0];
+      w[1] = q[1];
+      w[2] = q[2];
     }
-    if (mine) block_fma<S, K, NB>(cur, sh, tab, rc, xc, xstride, acc);
-    xc += 256;
+    block_fma<S, K, NB>(cur, sh, tab, rc, xc + i * 8, xstride, acc);
   }
 }
 
-// Blocks [ca, cb) of row r (a column range inside the staged chunk starting at
-// block cb0).  Rungs are non-decreasing along a row, so the range crosses at
-// most J rung segments; each runs a loop specialized for its rung.  Returns
-// the warp-wide sums in acc (every lane holds them).
 template <int NB>
-__device__ __forceinline__ void row_range(const GemvArgs &a, const uint64_t *tabs, const float *xs,
-                                          int64_t r, int ca, int cb, int cb0, int lane,
-                                          float (&acc)[NB]) {
-  const LayerArgs &p = a.p;
-  const int J = p.J;
-  const uint64_t roff = __ldg(p.row_off + r);
-  const uint32_t *base = p.stream + (roff >> 5);
-  const uint32_t rbit = (uint32_t)(roff & 31);
-  const int xstride = a.cw * 8;
-#pragma unroll
-  for (int b = 0; b < NB; ++b) acc[b] = 0.f;
-  uint32_t seg_bits = 0;  // bits of the row before block `lo`
-  int lo = 0;
-  for (int j = 0; j < J && lo < cb; ++j) {
-    const int hi = (j < J - 1) ? __ldg(p.brk + r * (J - 1) + j) : p.nb;
-    const int Lj = p.L[j];
-    const int s0 = max(lo, ca), s1 = min(hi, cb);
-    if (s0 < s1) {
-      const uint32_t bit0 = rbit + seg_bits + (uint32_t)(s0 - lo) * Lj;
-      const uint64_t *tab = tabs + p.slot[j] * 512;
-      const float *xc0 = xs + (s0 - cb0) * 8;
-      switch (p.code[j]) {
-#define SEEDQ_CASE(S_, K_)                                                                  \
-  case rung_code(S_, K_):                                                                   \
-    run_segment<S_, K_, NB>(base, bit0, s1 - s0, tab, xc0, xstride, lane, a.zero, acc);     \
+__device__ __forceinline__ void dispatch_cols(int code, const uint32_t *rowbuf, uint32_t &pos, int n,
+                                              const uint64_t *tab, const float *xc, int xstride,
+                                              uint32_t z, float (&acc)[NB]) {
+  switch (code) {
+#define SEEDQ_CASE(S_, K_)                                                   \
+  case rung_code(S_, K_):                                                    \
+    run_cols<S_, K_, NB>(rowbuf, pos, n, tab, xc, xstride, z, acc);          \
     break;
-        SEEDQ_FOR_EACH_RUNG(SEEDQ_CASE)
+    SEEDQ_FOR_EACH_RUNG(SEEDQ_CASE)
 #undef SEEDQ_CASE
-        default:
-          break;
-      }
-    }
-    seg_bits += (uint32_t)(hi - lo) * Lj;
+    default:
+      break;
+  }
+}
+
+// Bits of the lane's row before block x (rung j spans [bk[j-1], bk[j])).
+__device__ __forceinline__ uint32_t lane_bits_before(const int32_t *bk, int J, const int32_t *L,
+                                                     int nb, int x) {
+  uint32_t s = 0;
+  int lo = 0;
+  for (int j = 0; j < J; ++j) {
+    const int hi = (j < J - 1) ? bk[j] : nb;
+    s += (uint32_t)L[j] * (uint32_t)(min(max(x, lo), hi) - lo);
     lo = hi;
   }
+  return s;
+}
+
+// A piece of a round: blocks [ca, cb) of row group g of the round's tensor.
+struct Piece {
+  int64_t g;
+  int ca, cb;
+};
+
+// The stages of a round (pieces cut into ST-column stages, in order) dealt
+// round-robin to the CTA's warps; lane = row of the stage's row group.  Each
+// buffer slot carries the row data of the stage staged into it.  A warp's sums
+// go to comb[piece][warp][lane] whenever its next stage is in another piece.
+template <int NB>
+__device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t z,
+                                           const uint64_t *tabs, uint32_t *sbuf, float *xbuf,
+                                           int32_t *bk, const Piece *pcs, int np, int nst_total,
+                                           float *comb, int warp, int lane) {
+  using CF = Cfg<NB>;
+  const LayerArgs &p = T.p;
+  const int J = p.J, nb = p.nb;
+  if (warp >= nst_total) return;
+  const uint8_t *gstream = reinterpret_cast<const uint8_t *>(p.stream);
+  int piece_of[2] = {0, 0}, cs_of[2] = {0, 0}, ce_of[2] = {0, 0};
+  uint32_t pos0[2] = {0, 0};
+
+  auto issue = [&](int t, int sb) {
+    int pi = 0;
+    int nsp = (pcs[0].cb - pcs[0].ca + CF::ST - 1) / CF::ST;
+    while (t >= nsp && pi + 1 < np) {
+      t -= nsp;
+      ++pi;
+      nsp = (pcs[pi].cb - pcs[pi].ca + CF::ST - 1) / CF::ST;
+    }
+    const int cs = pcs[pi].ca + t * CF::ST, ce = min(pcs[pi].cb, cs + CF::ST);
+    const int64_t r0 = pcs[pi].g * 32;
+    const int64_t ridx = r0 + lane;
+    const int64_t row = __ldg(p.rowperm + (ridx < p.R ? ridx : r0));
+    const uint64_t roff = __ldg(p.row_off + row);
+    int32_t *mybk = bk + (sb * 32 + lane) * 8;
+    for (int j = 0; j < J - 1; ++j) mybk[j] = __ldg(p.brk + row * (J - 1) + j);
+    const uint64_t bit_cs = roff + lane_bits_before(mybk, J, p.L, nb, cs);
+    const uint64_t b_lo = (bit_cs >> 3) & ~(uint64_t)15;
+    uint64_t b_hi = (roff + lane_bits_before(mybk, J, p.L, nb, ce) + 96 + 7) >> 3;
+    b_hi = (b_hi + 15) & ~(uint64_t)15;
+    if (b_hi > T.stream_bytes) b_hi = T.stream_bytes & ~(uint64_t)15;
+    const int npc = b_hi > b_lo ? (int)min((uint64_t)CF::PIECES, (b_hi - b_lo) >> 4) : 0;
+    const uint32_t p0 = (uint32_t)(bit_cs - b_lo * 8);
+    if (sb) {
+      piece_of[1] = pi; cs_of[1] = cs; ce_of[1] = ce; pos0[1] = p0;
+    } else {
+      piece_of[0] = pi; cs_of[0] = cs; ce_of[0] = ce; pos0[0] = p0;
+    }
+    uint32_t *rows = sbuf + sb * 32 * CF::RW;
+    for (int i = 0; i < 16; ++i) {
+      const int r = 2 * i + (lane >> 4), pc = lane & 15;
+      const uint64_t blo = __shfl_sync(0xffffffffu, b_lo, r);
+      const int npr = __shfl_sync(0xffffffffu, npc, r);
+      if (pc < npr) cp_async16(rows + r * CF::RW + pc * 4, gstream + blo + 16 * pc);
+    }
+    float *xs = xbuf + sb * CF::ST * 8 * NB;
+    const int nq = (ce - cs) * 2;  // 16-byte pieces per batch column
+    for (int t2 = lane; t2 < n * nq; t2 += 32) {
+      const int b = t2 / nq, q = t2 - b * nq;
+      cp_async16(xs + b * CF::ST * 8 + q * 4, p.xperm + (int64_t)b * p.C + cs * 8 + q * 4);
+    }
+    cp_async_commit();
+  };
+
+  float acc[NB];
 #pragma unroll
-  for (int b = 0; b < NB; ++b) {
-    float v = acc[b];
+  for (int b = 0; b < NB; ++b) acc[b] = 0.f;
+  int acc_piece = -1;
+  issue(warp, 0);
+  int it = 0;
+  for (int t = warp; t < nst_total; t += kWarps, ++it) {
+    const int sb = it & 1;
+    if (t + kWarps < nst_total) {
+      issue(t + kWarps, sb ^ 1);
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
+    __syncwarp();
+    const int pi = sb ? piece_of[1] : piece_of[0];
+    const int cs = sb ? cs_of[1] : cs_of[0], ce = sb ? ce_of[1] : ce_of[0];
+    uint32_t pos = sb ? pos0[1] : pos0[0];
+    if (pi != acc_piece) {
+      if (acc_piece >= 0) {
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    acc[b] = v;
+        for (int b = 0; b < NB; ++b) comb[((acc_piece * kWarps + warp) * 32 + lane) * NB + b] += acc[b];
+      }
+#pragma unroll
+      for (int b = 0; b < NB; ++b) acc[b] = 0.f;
+      acc_piece = pi;
+    }
+    const int32_t *mybk = bk + (sb * 32 + lane) * 8;
+    const uint32_t *rowbuf = sbuf + sb * 32 * CF::RW + lane * CF::RW;
+    const float *xs = xbuf + sb * CF::ST * 8 * NB;
+    int jr = 0;
+    while (jr < J - 1 && mybk[jr] <= cs) ++jr;
+    int nxt = (jr < J - 1) ? mybk[jr] : nb;
+    int c = cs;
+    while (c < ce) {
+      const int jmin = __reduce_min_sync(0xffffffffu, jr), jmax = __reduce_max_sync(0xffffffffu, jr);
+      if (jmin == jmax) {
+        const int run_end = min((int)__reduce_min_sync(0xffffffffu, (unsigned)nxt), ce);
+        dispatch_cols<NB>(p.code[jmin], rowbuf, pos, run_end - c, tabs + p.slot[jmin] * 512,
+                          xs + (c - cs) * 8, CF::ST * 8, z, acc);
+        c = run_end;
+      } else {
+        // Rows at different rungs in this column: one pass per rung present.
+        for (int rr = jmin; rr <= jmax; ++rr) {
+          if (__any_sync(0xffffffffu, jr == rr) && jr == rr)
+            dispatch_cols<NB>(p.code[rr], rowbuf, pos, 1, tabs + p.slot[rr] * 512,
+                              xs + (c - cs) * 8, CF::ST * 8, z, acc);
+        }
+        c += 1;
+      }
+      while (jr < J - 1 && nxt <= c) {
+        ++jr;
+        nxt = (jr < J - 1) ? mybk[jr] : nb;
+      }
+    }
+    __syncwarp();
+  }
+  if (acc_piece >= 0) {
+#pragma unroll
+    for (int b = 0; b < NB; ++b) comb[((acc_piece * kWarps + warp) * 32 + lane) * NB + b] += acc[b];
   }
 }
 
 // Outlier epilogue: y_b[r] += sum_o W16[r, col_o] x_b[col_o] (Sec. 3.5).
-__device__ __forceinline__ float outlier_term(const GemvArgs &a, int64_t r, int b) {
+__device__ __forceinline__ float outlier_term(const TensorArgs &T, int64_t r, int b) {
   float s = 0.f;
-  for (int o = 0; o < a.p.n_out; ++o) {
-    const float w = __half2float(__ushort_as_half(a.p.out_vals[r * a.p.n_out + o]));
-    s = __fmaf_rn(w, bf16_to_f32(a.x[(int64_t)b * a.p.C + a.p.out_cols[o]]), s);
+  for (int o = 0; o < T.p.n_out; ++o) {
+    const float w = __half2float(__ushort_as_half(T.p.out_vals[r * T.p.n_out + o]));
+    s = __fmaf_rn(w, bf16_to_f32(T.x[(int64_t)b * T.p.C + T.p.out_cols[o]]), s);
   }
   return s;
 }
 
 template <int NB>
-__global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ GemvArgs a) {
+__global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ MultiArgs a) {
+  using CF = Cfg<NB>;
   extern __shared__ __align__(16) uint64_t smem[];
-  const LayerArgs &p = a.p;
   uint64_t *tabs = smem;
-  float *xs = reinterpret_cast<float *>(smem + p.nslots * 512);
-  float *racc = xs + NB * a.cw * 8;               // rt x NB row accumulators
-  float *slot = racc + a.rt * NB;                 // kWarps x 2 x NB partial sums
-  int *slot_row = reinterpret_cast<int *>(slot + kWarps * 2 * NB);
-  {
-    const uint4 *src = reinterpret_cast<const uint4 *>(p.tables);
-    uint4 *dst = reinterpret_cast<uint4 *>(tabs);
-    for (int i = threadIdx.x; i < p.nslots * 256; i += kThreads) dst[i] = __ldg(src + i);
-  }
+  uint8_t *wbase = reinterpret_cast<uint8_t *>(smem + kTableSlots * 512);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  for (int tile = blockIdx.x; tile < a.ntiles; tile += gridDim.x) {
-    const int64_t r_lo = (int64_t)tile * a.rt;
-    const int nr = (int)min((int64_t)a.rt, p.R - r_lo);
-    for (int i = threadIdx.x; i < nr * NB; i += kThreads) racc[i] = 0.f;
-    for (int ch = 0; ch < a.nchunks; ++ch) {
-      const int cb0 = ch * a.cw, cb1 = min(cb0 + a.cw, p.nb), ncb = cb1 - cb0;
-      __syncthreads();
-      // Stage the chunk's activations in permuted order (0 at outlier columns):
-      // coalesced reads of x and of the inverse permutation, scattered into
-      // shared memory, so no load waits on another.
-      for (int col0 = threadIdx.x; col0 < p.C; col0 += 4 * kThreads) {
-        int pos[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int col = col0 + u * kThreads;
-          pos[u] = (col < p.C) ? __ldg(p.invperm + col) - cb0 * 8 : -1;
-        }
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int col = col0 + u * kThreads;
-          if (pos[u] >= 0 && pos[u] < ncb * 8) {
-            bool outl = false;
-            for (int o = 0; o < p.n_out; ++o) outl |= (p.out_cols[o] == col);
-            for (int b = 0; b < a.n; ++b)
-              xs[b * a.cw * 8 + pos[u]] = outl ? 0.f : bf16_to_f32(__ldg(a.x + (int64_t)b * p.C + col));
+  uint8_t *mine = wbase + warp * CF::WARP_BYTES;
+  uint32_t *sbuf = reinterpret_cast<uint32_t *>(mine);
+  float *xbuf = reinterpret_cast<float *>(mine + CF::STREAM_WORDS * 4);
+  int32_t *bk = reinterpret_cast<int32_t *>(mine + CF::STREAM_WORDS * 4 + CF::XFLOATS * 4);
+  float *comb = reinterpret_cast<float *>(wbase + kWarps * CF::WARP_BYTES);  // RG x kWarps x 32 x NB
+  int *flag = reinterpret_cast<int *>(comb + CF::RG * kWarps * 32 * NB);
+  {
+    // The jump tables depend only on S, so any tensor's copy serves all.
+    const uint4 *src = reinterpret_cast<const uint4 *>(a.t[0].p.tables);
+    uint4 *dst = reinterpret_cast<uint4 *>(tabs);
+    for (int i = threadIdx.x; i < kTableSlots * 256; i += kThreads) dst[i] = __ldg(src + i);
+  }
+  const int cta = blockIdx.x;
+  const int64_t u0 = a.cta_begin[cta], u1 = a.cta_begin[cta + 1];
+  int64_t u = u0;
+  bool first = true;
+  while (u < u1) {
+    int ti = 0;
+    while (ti + 1 < a.nt && a.t[ti + 1].ubegin <= u) ++ti;
+    const TensorArgs &T = a.t[ti];
+    const LayerArgs &p = T.p;
+    const int64_t tend = (ti + 1 < a.nt) ? a.t[ti + 1].ubegin : a.cta_begin[a.ctas];
+    const int64_t rend = min(u1, tend);
+    // The next round: up to RG row groups of this tensor.
+    Piece pcs[CF::RG];
+    int np = 0, nst_total = 0;
+    int64_t uu = u;
+    while (uu < rend && np < CF::RG) {
+      const int64_t lu = uu - T.ubegin;
+      const int64_t g = lu / p.nb;
+      const int ca = (int)(lu - g * p.nb);
+      const int cb = (int)min((int64_t)p.nb, ca + (rend - uu));
+      pcs[np] = Piece{g, ca, cb};
+      nst_total += (cb - ca + CF::ST - 1) / CF::ST;
+      ++np;
+      uu += cb - ca;
+    }
+    for (int i = threadIdx.x; i < np * kWarps * 32 * NB; i += kThreads) comb[i] = 0.f;
+    __syncthreads();
+    warp_round<NB>(T, a.n, a.zero, tabs, sbuf, xbuf, bk, pcs, np, nst_total, comb, warp, lane);
+    __syncthreads();
+    for (int k = 0; k < np; ++k) {
+      const int64_t g = pcs[k].g, r0 = g * 32;
+      const bool full = (pcs[k].ca == 0 && pcs[k].cb == p.nb);
+      const int sidx = (k == 0 && first) ? 0 : 1;
+      for (int i = threadIdx.x; i < 32 * NB; i += kThreads) {
+        float v = 0.f;
+        for (int w = 0; w < kWarps; ++w) v += comb[(k * kWarps + w) * 32 * NB + i];
+        const int ln = i / NB, b = i - ln * NB;
+        if (full) {
+          if (r0 + ln < p.R && b < a.n) {
+            const int64_t rr = __ldg(p.rowperm + r0 + ln);
+            T.y[(int64_t)b * p.R + rr] = v + outlier_term(T, rr, b);
           }
+        } else {
+          p.slots[((int64_t)cta * 2 + sidx) * 32 * kMaxBatch + i] = v;
         }
       }
-      if (threadIdx.x < kWarps * 2) slot_row[threadIdx.x] = -1;
-      __syncthreads();
-      // This warp's equal share of the tile's (row, block) pairs in the chunk.
-      const int64_t work = (int64_t)nr * ncb;
-      const int64_t wb0 = work * warp / kWarps, wb1 = work * (warp + 1) / kWarps;
-      int64_t wb = wb0;
-      while (wb < wb1) {
-        const int rr = (int)(wb / ncb);
-        const int c0 = (int)(wb - (int64_t)rr * ncb);
-        const int c1 = (int)min((int64_t)ncb, c0 + (wb1 - wb));
-        float acc[NB];
-        row_range<NB>(a, tabs, xs, r_lo + rr, cb0 + c0, cb0 + c1, cb0, lane, acc);
-        if (lane == 0) {
-          if (c0 == 0 && c1 == ncb) {  // whole row of the chunk: sole writer
-#pragma unroll
-            for (int b = 0; b < NB; ++b) racc[rr * NB + b] += acc[b];
-          } else {
-            const int s = (wb == wb0) ? 0 : 1;
-            slot_row[warp * 2 + s] = rr;
-#pragma unroll
-            for (int b = 0; b < NB; ++b) slot[(warp * 2 + s) * NB + b] = acc[b];
-          }
+      if (!full) {
+        const int64_t gu = T.ubegin + g * p.nb;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+          __threadfence();
+          const int cf = cta_of(a, gu), cl = cta_of(a, gu + p.nb - 1);
+          const int old = atomicAdd(p.counters + g, 1);
+          *flag = (old == cl - cf) ? 1 : 0;
         }
-        wb += c1 - c0;
-      }
-      __syncthreads();
-      // Rows cut by range boundaries: add the partial sums in warp order.
-      for (int rr = threadIdx.x; rr < nr; rr += kThreads) {
-        for (int sidx = 0; sidx < kWarps * 2; ++sidx) {
-          if (slot_row[sidx] == rr) {
-            for (int b = 0; b < NB; ++b) racc[rr * NB + b] += slot[sidx * NB + b];
+        __syncthreads();
+        if (*flag) {
+          __threadfence();
+          const int cf = cta_of(a, gu), cl = cta_of(a, gu + p.nb - 1);
+          for (int i = threadIdx.x; i < 32 * NB; i += kThreads) {
+            float v = 0.f;
+            for (int c2 = cf; c2 <= cl; ++c2) {
+              const int s2 = (a.cta_begin[c2] >= gu) ? 0 : 1;
+              v += __ldcg(p.slots + ((int64_t)c2 * 2 + s2) * 32 * kMaxBatch + i);
+            }
+            const int ln = i / NB, b = i - ln * NB;
+            if (r0 + ln < p.R && b < a.n) {
+              const int64_t rr = __ldg(p.rowperm + r0 + ln);
+              T.y[(int64_t)b * p.R + rr] = v + outlier_term(T, rr, b);
+            }
           }
+          if (threadIdx.x == 0) p.counters[g] = 0;
         }
+        __syncthreads();
       }
     }
     __syncthreads();
-    for (int i = threadIdx.x; i < nr * a.n; i += kThreads) {
-      const int rr = i / a.n, b = i - rr * a.n;
-      const int64_t r = r_lo + rr;
-      a.y[(int64_t)b * p.R + r] = racc[rr * NB + b] + outlier_term(a, r, b);
+    first = false;
+    u = uu;
+  }
+}
+
+// Activations in permuted column order, zero at outlier columns (their
+// contribution is added exactly by the epilogue): xperm[b][p] = x_b[perm[p]].
+__global__ void k_xperm(const __grid_constant__ MultiArgs a) {
+  for (int ti = 0; ti < a.nt; ++ti) {
+    const TensorArgs &T = a.t[ti];
+    const LayerArgs &p = T.p;
+    const int64_t total = (int64_t)a.n * p.C;
+    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
+         t += (int64_t)gridDim.x * blockDim.x) {
+      const int64_t b = t / p.C;
+      const int pc = (int)(t - b * p.C);
+      const int col = __ldg(p.perm + pc);
+      bool outl = false;
+      for (int o = 0; o < p.n_out; ++o) outl |= (p.out_cols[o] == col);
+      p.xperm[t] = outl ? 0.f : bf16_to_f32(__ldg(T.x + b * p.C + col));
     }
-    __syncthreads();
   }
 }
 
 template <int NB>
-static size_t smem_bytes(int nslots, int cw, int rt) {
-  return sizeof(uint64_t) * 512 * nslots + sizeof(float) * NB * cw * 8 + sizeof(float) * rt * NB +
-         sizeof(float) * kWarps * 2 * NB + sizeof(int) * kWarps * 2;
+static size_t smem_bytes() {
+  return sizeof(uint64_t) * 512 * kTableSlots + (size_t)kWarps * Cfg<NB>::WARP_BYTES +
+         sizeof(float) * Cfg<NB>::RG * kWarps * 32 * NB + 16;
+}
+
+// Cost-balanced ranges of the units of all tensors, one per CTA.
+static void partition(const seedq_layer *const *layers, int nt, MultiArgs &a) {
+  int64_t U = 0;
+  double total = 0.0;
+  for (int i = 0; i < nt; ++i) {
+    const seedq_layer *L = layers[i];
+    const int64_t G = (L->args.R + 31) / 32;
+    a.t[i].ubegin = U;
+    U += G * L->args.nb;
+    total += L->h_gcost[G];
+  }
+  int ctas = layers[0]->max_ctas;
+  if (ctas > kMaxCtas) ctas = kMaxCtas;
+  if (U < ctas) ctas = (int)U;
+  a.ctas = ctas;
+  a.cta_begin[0] = 0;
+  a.cta_begin[ctas] = U;
+  int ti = 0;
+  double tbase = 0.0;  // cost of the tensors before ti
+  for (int c = 1; c < ctas; ++c) {
+    const double target = total * c / ctas;
+    const seedq_layer *L = layers[ti];
+    int64_t G = (L->args.R + 31) / 32;
+    while (ti + 1 < nt && tbase + L->h_gcost[G] <= target) {
+      tbase += L->h_gcost[G];
+      L = layers[++ti];
+      G = (L->args.R + 31) / 32;
+    }
+    const double lt = target - tbase;
+    int64_t lo = 0, hi = G - 1;  // last group with h_gcost[g] <= lt
+    while (lo < hi) {
+      const int64_t mid = (lo + hi + 1) / 2;
+      if (L->h_gcost[mid] <= lt) lo = mid;
+      else hi = mid - 1;
+    }
+    const int64_t g = lo;
+    const int J = L->args.J, Jm1 = J > 1 ? J - 1 : 1, nb = L->args.nb;
+    const int32_t *b = L->h_repbk + g * Jm1;
+    double acc = L->h_gcost[g];
+    int col = nb, clo = 0;
+    for (int j = 0; j < J; ++j) {
+      const int chi = (j < J - 1) ? b[j] : nb;
+      const double seg = L->h_cost[j] * (chi - clo);
+      if (acc + seg > lt) {
+        col = clo + (int)((lt - acc) / L->h_cost[j]);
+        break;
+      }
+      acc += seg;
+      clo = chi;
+    }
+    int64_t u = a.t[ti].ubegin + g * nb + col;
+    if (u <= a.cta_begin[c - 1]) u = a.cta_begin[c - 1] + 1;
+    if (u > U - (ctas - c)) u = U - (ctas - c);
+    a.cta_begin[c] = u;
+  }
 }
 
 template <int NB>
-static seedq_status launch(const seedq_layer *L, const uint16_t *x, int n, float *y,
-                           cudaStream_t st) {
-  int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  GemvArgs a;
-  a.p = L->args;
-  a.x = x;
-  a.y = y;
-  a.n = n;
-  a.zero = 0u;
-  const int cw_max = kXBytes / (int)sizeof(float) / 8 / NB;
-  a.cw = L->args.nb < cw_max ? L->args.nb : cw_max;
-  a.nchunks = (L->args.nb + a.cw - 1) / a.cw;
-  int64_t rt = (L->args.R + sms - 1) / sms;
-  if (rt * NB > kAccFloats) rt = kAccFloats / NB;
-  a.rt = (int)rt;
-  a.ntiles = (int)((L->args.R + rt - 1) / rt);
-  const size_t smem = smem_bytes<NB>(L->args.nslots, a.cw, a.rt);
+static seedq_status launch(const seedq_layer *const *layers, int nt, const uint16_t *const *x, int n,
+                           float *const *y, cudaStream_t st) {
+  MultiArgs args;
+  MultiArgs *a = &args;
+  a->nt = nt;
+  a->n = n;
+  a->zero = 0u;
+  for (int i = 0; i < nt; ++i) {
+    a->t[i].p = layers[i]->args;
+    a->t[i].x = x[i];
+    a->t[i].y = y[i];
+    a->t[i].stream_bytes = layers[i]->stream_bytes;
+  }
+  partition(layers, nt, *a);
   static bool attr_set = false;
+  seedq_status rc = SEEDQ_OK;
   if (!attr_set) {
-    SEEDQ_CUDA(cudaFuncSetAttribute(k_gemv<NB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    (int)smem_bytes<NB>(kMaxJ, cw_max, kAccFloats / NB)));
-    attr_set = true;
+    const cudaError_t e = cudaFuncSetAttribute(k_gemv<NB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               (int)smem_bytes<NB>());
+    if (e != cudaSuccess) rc = cuda_fail(e);
+    else attr_set = true;
   }
-  const int grid = a.ntiles < sms ? a.ntiles : sms;
-  k_gemv<NB><<<grid, kThreads, smem, st>>>(a);
-  SEEDQ_CUDA(cudaGetLastError());
-  return SEEDQ_OK;
+  if (rc == SEEDQ_OK) {
+    int64_t total = 0;
+    for (int i = 0; i < nt; ++i) total += (int64_t)n * layers[i]->args.C;
+    const int64_t want = (total + 255) / 256;
+    const int g = (int)(want < (int64_t)layers[0]->max_ctas * 8 ? want : (int64_t)layers[0]->max_ctas * 8);
+    k_xperm<<<g, 256, 0, st>>>(*a);
+    cudaError_t e = cudaGetLastError();
+    if (e == cudaSuccess) {
+      k_gemv<NB><<<a->ctas, kThreads, smem_bytes<NB>(), st>>>(*a);
+      e = cudaGetLastError();
+    }
+    if (e != cudaSuccess) rc = cuda_fail(e);
+  }
+  return rc;
 }
 
-// The fused kernel keeps no global scratch (partial sums live in shared memory).
-int64_t gemv_partial_elems(const seedq_layer *, int) { return 0; }
+static seedq_status gemm_multi(const seedq_layer *const *layers, int nt, const uint16_t *const *X,
+                               int n, float *const *Y, cudaStream_t st) {
+  if (!layers || !X || !Y || nt < 1 || nt > kMaxTensors || n < 1 || n > kMaxBatch)
+    return SEEDQ_ERR_INVALID_ARG;
+  for (int i = 0; i < nt; ++i) {
+    if (!layers[i] || !X[i] || !Y[i] || n > layers[i]->max_batch) return SEEDQ_ERR_INVALID_ARG;
+    if (!layers[i]->args.stream) return SEEDQ_ERR_STREAM;
+  }
+  switch (batch_template(n)) {
+    case 1: return launch<1>(layers, nt, X, n, Y, st);
+    case 2: return launch<2>(layers, nt, X, n, Y, st);
+    case 4: return launch<4>(layers, nt, X, n, Y, st);
+    case 8: return launch<8>(layers, nt, X, n, Y, st);
+    default: return launch<16>(layers, nt, X, n, Y, st);
+  }
+}
 
 }  // namespace seedq
 
@@ -295,22 +558,17 @@ extern "C" {
 
 seedq_status seedq_gemm_small_batch(const seedq_layer *L, const uint16_t *X, int32_t n, float *Y,
                                     void *cuda_stream) {
-  if (!L || !X || !Y || n < 1 || n > L->max_batch) return SEEDQ_ERR_INVALID_ARG;
-  if (!L->args.stream) return SEEDQ_ERR_STREAM;
-  cudaStream_t st = (cudaStream_t)cuda_stream;
-  switch (batch_template(n)) {
-    case 1: return launch<1>(L, X, n, Y, st);
-    case 2: return launch<2>(L, X, n, Y, st);
-    case 4: return launch<4>(L, X, n, Y, st);
-    case 8: return launch<8>(L, X, n, Y, st);
-    default: return launch<16>(L, X, n, Y, st);
-  }
+  return gemm_multi(&L, 1, &X, n, &Y, (cudaStream_t)cuda_stream);
 }
 
 seedq_status seedq_gemv(const seedq_layer *L, const uint16_t *x, float *y, void *cuda_stream) {
-  if (!L || !x || !y) return SEEDQ_ERR_INVALID_ARG;
-  if (!L->args.stream) return SEEDQ_ERR_STREAM;
-  return launch<1>(L, x, 1, y, (cudaStream_t)cuda_stream);
+  return gemm_multi(&L, 1, &x, 1, &y, (cudaStream_t)cuda_stream);
+}
+
+seedq_status seedq_gemm_multi(const seedq_layer *const *layers, int32_t count,
+                              const uint16_t *const *X, int32_t n, float *const *Y,
+                              void *cuda_stream) {
+  return gemm_multi(layers, count, X, n, Y, (cudaStream_t)cuda_stream);
 }
 
 }  // extern "C"

@@ -56,6 +56,34 @@ __global__ void k_perm(const float *__restrict__ a, int C, int32_t *__restrict__
   if (i < C) perm[rank] = i;
 }
 
+// Row order for the fused kernel: rows with equal or nearby rung breakpoints
+// share a warp.  Breakpoints are monotone in the row factor (imp = abar * rho),
+// so rows are ranked by decreasing rho (ties by index); with no row factor every
+// row has the same breakpoints and the natural order is kept.
+__global__ void k_rowrank(const double *__restrict__ rho, int R, int32_t *__restrict__ rowperm) {
+  __shared__ double tile[1024];
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  const double ri = (i < R) ? rho[i] : 0.0;
+  int rank = 0;
+  for (int base = 0; base < R; base += 1024) {
+    __syncthreads();
+    for (int t = threadIdx.x; t < 1024; t += blockDim.x) tile[t] = (base + t < R) ? rho[base + t] : 0.0;
+    __syncthreads();
+    const int n = min(1024, R - base);
+    for (int t = 0; t < n; ++t) {
+      const double v = tile[t];
+      rank += (v > ri || (v == ri && base + t < i)) ? 1 : 0;
+    }
+  }
+  if (i < R) rowperm[rank] = i;
+}
+
+__global__ void k_iota(int64_t n, int32_t *__restrict__ out) {
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x)
+    out[i] = (int32_t)i;
+}
+
 __global__ void k_invperm(const int32_t *__restrict__ perm, int C, int32_t *__restrict__ inv) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i < C) inv[perm[i]] = i;
@@ -278,12 +306,60 @@ static void free_layer(seedq_layer *L) {
   cudaFree(L->d_tables);
   cudaFree(L->d_flags);
   cudaFree(L->d_summary);
-  cudaFree(L->d_partials);
+  cudaFree(L->d_rowperm);
+  cudaFree(L->d_counters);
+  cudaFree(L->d_slots);
+  cudaFree(L->d_xperm);
+  free(L->h_gcost);
+  free(L->h_repbk);
 
   free(L);
 }
 
-int64_t gemv_partial_elems(const seedq_layer *L, int max_batch);  // gemv.cu
+
+// Host-side cost profile of the tensor for the fused kernel's work partition.
+// Units are (row group, block) pairs in row-group-major order; a unit's cost is
+// modeled by the reconstruction work of its rung (8 (k+1) logic/FMA steps plus
+// a fixed per-block part), taken from the first row of the group in the
+// kernel's row order.  Kept: the cumulative cost per row group and those rows'
+// breakpoints, from which any cost target maps back to a (group, block) unit.
+static seedq_status build_costs(seedq_layer *L, cudaStream_t st) {
+  const int64_t R = L->args.R;
+  const int J = L->args.J, Jm1 = J > 1 ? J - 1 : 1;
+  const int64_t G = (R + 31) / 32;
+  int32_t *rowperm = (int32_t *)malloc(sizeof(int32_t) * R);
+  int32_t *brk = (int32_t *)malloc(sizeof(int32_t) * R * Jm1);
+  L->h_gcost = (double *)malloc(sizeof(double) * (G + 1));
+  L->h_repbk = (int32_t *)malloc(sizeof(int32_t) * G * Jm1);
+  seedq_status rc = SEEDQ_OK;
+  if (!rowperm || !brk || !L->h_gcost || !L->h_repbk) rc = SEEDQ_ERR_NOMEM;
+  cudaError_t e = cudaSuccess;
+  if (rc == SEEDQ_OK) e = cudaMemcpyAsync(rowperm, L->d_rowperm, sizeof(int32_t) * R, cudaMemcpyDeviceToHost, st);
+  if (rc == SEEDQ_OK && e == cudaSuccess && J > 1)
+    e = cudaMemcpyAsync(brk, L->d_brk, sizeof(int32_t) * R * Jm1, cudaMemcpyDeviceToHost, st);
+  if (rc == SEEDQ_OK && e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) rc = cuda_fail(e);
+  if (rc == SEEDQ_OK) {
+    for (int j = 0; j < J; ++j) L->h_cost[j] = 8.0 * (L->k[j] + 1) + 40.0;
+    L->h_gcost[0] = 0.0;
+    for (int64_t g = 0; g < G; ++g) {
+      const int32_t *b = brk + (int64_t)rowperm[g * 32] * Jm1;
+      int32_t *rb = L->h_repbk + g * Jm1;
+      double c = 0.0;
+      int lo = 0;
+      for (int j = 0; j < J; ++j) {
+        const int hi = (j < J - 1) ? b[j] : L->args.nb;
+        if (j < J - 1) rb[j] = b[j];
+        c += L->h_cost[j] * (hi - lo);
+        lo = hi;
+      }
+      L->h_gcost[g + 1] = L->h_gcost[g] + c;
+    }
+  }
+  free(rowperm);
+  free(brk);
+  return rc;
+}
 
 }  // namespace seedq
 
@@ -363,20 +439,16 @@ seedq_status seedq_layer_prepare(const seedq_layer_desc *d, const seedq_schedule
   L->tie_count = d->tie_count;
   L->max_batch = mb;
   cudaGetDevice(&L->device);
-  int nslots = 0;
+  // One jump-table slot per supported seed width (8, 10, ..., 16); the tables
+  // depend only on S, so every layer's table set is the same.
+  const int nslots = kTableSlots;
+  for (int t = 0; t < nslots; ++t) L->slot_S[t] = 8 + 2 * t;
   for (int j = 0; j < J; ++j) {
     L->S[j] = s->rungs[j].S;
     L->k[j] = s->rungs[j].k;
     L->args.L[j] = L->S[j] + 4 * L->k[j] + 4;
     L->args.code[j] = rung_code(L->S[j], L->k[j]);
-    int slot = -1;
-    for (int t = 0; t < nslots; ++t)
-      if (L->slot_S[t] == L->S[j]) slot = t;
-    if (slot < 0) {
-      slot = nslots;
-      L->slot_S[nslots++] = L->S[j];
-    }
-    L->args.slot[j] = slot;
+    L->args.slot[j] = (L->S[j] - 8) / 2;
     if (j + 1 < J) L->theta[j] = s->theta[j];
   }
   L->args.nslots = nslots;
@@ -420,11 +492,24 @@ seedq_status seedq_layer_prepare(const seedq_layer_desc *d, const seedq_schedule
     cudaFree(dS);
     if (e != cudaSuccess) { free_layer(L); return cuda_fail(e); }
   }
-  L->partial_elems = gemv_partial_elems(L, mb);
-  if (L->partial_elems) ALLOC(L->d_partials, sizeof(float) * L->partial_elems);
+  {
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    L->max_ctas = sms > 0 ? sms : 1;
+  }
+  const int64_t ngroups = (R + 31) / 32;
+  ALLOC(L->d_rowperm, sizeof(int32_t) * R);
+  ALLOC(L->d_counters, sizeof(int32_t) * ngroups);
+  ALLOC(L->d_slots, sizeof(float) * L->max_ctas * 2 * 32 * kMaxBatch);
+  ALLOC(L->d_xperm, sizeof(float) * C * mb);
 
 #undef ALLOC
   L->args.perm = L->d_perm;
+  L->args.rowperm = L->d_rowperm;
+  L->args.counters = L->d_counters;
+  L->args.slots = L->d_slots;
+  L->args.xperm = L->d_xperm;
   L->args.invperm = L->d_invperm;
   L->args.brk = L->d_brk;
   L->args.row_off = L->d_row_off;
@@ -458,6 +543,15 @@ seedq_status seedq_layer_prepare(const seedq_layer_desc *d, const seedq_schedule
     }
     k_scan<<<1, 1024, 0, st>>>(R, J, nb, J > 1 ? s->j_tie : -1, d->tie_count, dL, L->d_brk,
                                L->d_tcnt, L->d_row_off, L->d_summary);
+    bool rho_uniform = true;
+    if (d->rho)
+      for (int64_t r = 1; r < R; ++r) rho_uniform &= (d->rho[r] == d->rho[0]);
+    if (rho_uniform || R > 65536) {
+      k_iota<<<(int)((R + 255) / 256 < 4096 ? (R + 255) / 256 : 4096), 256, 0, st>>>(R, L->d_rowperm);
+    } else {
+      k_rowrank<<<(int)((R + 255) / 256), 256, 0, st>>>(L->d_rho, (int)R, L->d_rowperm);
+    }
+    if (e == cudaSuccess) e = cudaMemsetAsync(L->d_counters, 0, sizeof(int32_t) * ngroups, st);
     if (e == cudaSuccess) e = cudaGetLastError();
   }
   uint64_t summary[2] = {0, 0};
@@ -475,6 +569,13 @@ seedq_status seedq_layer_prepare(const seedq_layer_desc *d, const seedq_schedule
     return rc;
   }
   L->total_bits = summary[1];
+  {
+    seedq_status prc = build_costs(L, st);
+    if (prc != SEEDQ_OK) {
+      free_layer(L);
+      return prc;
+    }
+  }
   // The plan's fp32 copies of a and rho are no longer needed.
   cudaFree(L->d_a_in);
   L->d_a_in = nullptr;

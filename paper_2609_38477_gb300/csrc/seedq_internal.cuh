@@ -12,6 +12,7 @@ constexpr int kMaxJ = 9;         // hull rungs (App. B.3: four to eight on the p
 constexpr int kMaxOutliers = 16; // FP16 outlier columns (Sec. 3.5 stores four)
 constexpr int kMaxBatch = 16;    // decode batch of seedq_gemm_small_batch
 constexpr int kMaxCols = 65536;
+constexpr int kTableSlots = 5;   // jump tables for S = 8, 10, 12, 14, 16
 
 // Supported rungs: S in {8,10,12,14,16}, k in {2..6} (the paper's grid, Sec. 3.1,
 // at the even seed widths its Table "Rung grids" uses).
@@ -37,6 +38,10 @@ struct LayerArgs {
   const int32_t *perm;      // C: block c holds columns perm[8c..8c+7]
   const int32_t *invperm;   // C: position of column j in the permuted order
   const uint16_t *out_vals; // R x n_out binary16
+  const int32_t *rowperm;   // R: order in which rows are grouped 32 to a warp
+  float *xperm;             // max_batch x C: activations in permuted column order
+  int32_t *counters;        // row groups: arrivals of partial sums (0 between calls)
+  float *slots;             // max_ctas x 2 x 32 x 16 partial sums of row groups
   uint32_t *flags;
   int64_t R, C;
   int32_t nb;               // C / 8 blocks per row
@@ -70,12 +75,18 @@ struct seedq_layer {
   float *d_rho_in, *d_a_in;
   int32_t *d_brk;
   int32_t *d_tcnt;
+  int32_t *d_rowperm;
+  int32_t *d_counters;
+  float *d_slots;
+  float *d_xperm;
+  int32_t max_ctas;      // CTAs of the fused kernel (one per SM)
+  double *h_gcost;       // host: cumulative modeled cost per row group (G + 1)
+  int32_t *h_repbk;      // host: breakpoints of each row group's first row (G x (J-1))
+  double h_cost[seedq::kMaxJ];  // modeled cost of one block per rung
   uint64_t *d_row_off;
   uint64_t *d_tables;
   uint32_t *d_flags;
   uint64_t *d_summary;   // [0] total tied blocks, [1] total bits
-  float *d_partials;     // split-K partial sums
-  int64_t partial_elems;
   // bound stream (caller-owned)
   const void *stream;
   uint64_t stream_bytes;

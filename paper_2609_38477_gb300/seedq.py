@@ -60,6 +60,8 @@ SIGNATURES = {
     "seedq_decode_rows": (C.c_int, [C.c_void_p, C.c_int64, C.c_int64, C.c_void_p, C.c_void_p]),
     "seedq_gemv": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
     "seedq_gemm_small_batch": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p]),
+    "seedq_gemm_multi": (C.c_int, [C.POINTER(C.c_void_p), C.c_int32, C.POINTER(C.c_void_p),
+                                   C.c_int32, C.POINTER(C.c_void_p), C.c_void_p]),
     "seedq_layer_rung_map": (C.c_int, [C.c_void_p, C.c_int64, C.c_int64, C.c_void_p]),
     "seedq_layer_perm": (C.c_int, [C.c_void_p, C.c_void_p]),
     "seedq_layer_row_offsets": (C.c_int, [C.c_void_p, C.c_void_p]),
@@ -225,3 +227,12 @@ def row_plan_static(abar, rho, rows: int, nb: int, rungs, theta, j_tie: int, q: 
     _check(lib().seedq_row_plan_static(_ptr(abar), _ptr(rho), rows, nb, C.byref(sched), tie_count,
                                        _ptr(brk), _ptr(row_off), _ptr(summary), _stream(stream)),
            "seedq_row_plan_static")
+
+
+def gemm_multi(layers, X, n: int, Y, stream=None):
+    """seedq_gemm_multi: Y[i] = X[i] W_hat_i^T for several layers in one launch."""
+    cnt = len(layers)
+    lh = (C.c_void_p * cnt)(*[l.h.value for l in layers])
+    xh = (C.c_void_p * cnt)(*[_ptr(x) for x in X])
+    yh = (C.c_void_p * cnt)(*[_ptr(y) for y in Y])
+    _check(lib().seedq_gemm_multi(lh, cnt, xh, n, yh, _stream(stream)), "seedq_gemm_multi")

@@ -198,24 +198,28 @@ def test_full_size_sampled(name):
     torch.cuda.synchronize()
     rng = np.random.default_rng(sum(map(ord, name)))
     worst = 0.0
+    # Every batch size of the workload, each as the benchmark runs it: all
+    # tensors through seedq_gemm_multi, eight per launch.
+    Ys = {}
+    xbs = {i: W.x_bf16(w, i, nbmax) for i in range(len(w.tensors))}
+    xds = {i: x_dev(xbs[i]) for i in range(len(w.tensors))}
+    for n in w.batches:
+        Ys[n] = [torch.empty((n, t.R), dtype=torch.float32, device="cuda") for t in w.tensors]
+        for c0 in range(0, len(gts), 8):
+            idx = list(range(c0, min(c0 + 8, len(gts))))
+            Q().gemm_multi([gts[i].layer for i in idx], [xds[i][:n] for i in idx], n,
+                           [Ys[n][i] for i in idx])
+    torch.cuda.synchronize()
     for i, gt in enumerate(gts):
         t = w.tensors[i]
-        # Batch sizes of the workload on a rotating subset, batch 1 everywhere.
-        batches = [1] + ([n for n in w.batches if n > 1] if i % 7 in (0, 4, 6) else [])
-        xb = W.x_bf16(w, i, max(batches))
-        xd = x_dev(xb)
-        Y = torch.empty((max(batches), t.R), dtype=torch.float32, device="cuda")
+        xb = xbs[i]
         rows = sorted({int(rng.integers(0, t.R)), t.R - 1})
         ot = otensor(w, i)
         key = W.payload_key(w, i)
         for r in rows:
             assert np.array_equal(gt.layer.rung_map(r, 1), ot.rung_rows(s, d["tie_count"][i], r, 1))
-        for n in batches:
-            if n == 1:
-                gt.layer.gemv(xd[:1], Y[0])
-            else:
-                gt.layer.gemm_small_batch(xd[:n], n, Y[:n])
-            Yh = Y[:n].cpu().numpy()
+        for n in w.batches:
+            Yh = Ys[n][i].cpu().numpy()
             for r in rows:
                 y64, yabs = ot.synth_gemv(s, d["tie_count"][i], key, xb[:n], r, 1)
                 worst = max(worst, check_y(Yh[:, r], y64[:, 0], yabs[:, 0]))
@@ -369,3 +373,28 @@ def test_api_errors_and_determinism():
     with pytest.raises(Qm.SeedQError) as e:
         Qm.Layer(R, Cc, a, rh, s2.rungs, s2.theta, 0, 0.0, tied + 1)
     assert e.value.status == 3
+
+
+@pytest.mark.parametrize("name", ["c1", "c2"])
+def test_layer_set_multi_launch(name):
+    """The benchmark's step: all seven tensors in one seedq_gemm_multi launch,
+    every output row checked against the oracle, at each batch size."""
+    w = W.WORKLOADS[name]
+    d, s = load(name)
+    nbmax = max(w.batches)
+    gts = [G().bind(G().prepare_tensor(w, i, d, max_batch=nbmax)) for i in range(len(w.tensors))]
+    xbs = [W.x_bf16(w, i, nbmax) for i in range(len(w.tensors))]
+    xds = [x_dev(x) for x in xbs]
+    ref = [otensor(w, i).synth_gemv(s, d["tie_count"][i], W.payload_key(w, i), xbs[i])
+           for i in range(len(w.tensors))]
+    for n in w.batches:
+        Ys = [torch.empty((n, t.R), dtype=torch.float32, device="cuda") for t in w.tensors]
+        Q().gemm_multi([g.layer for g in gts], [x[:n] for x in xds], n, Ys)
+        torch.cuda.synchronize()
+        for i in range(len(gts)):
+            Yh = Ys[i].cpu().numpy()
+            for b in range(n):
+                check_y(Yh[b], ref[i][0][b], ref[i][1][b])
+    for g in gts:
+        assert g.layer.device_error() == 0
+        g.layer.release()
