@@ -280,13 +280,22 @@ __device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t 
                           xs + (c - cs) * 8, CF::ST * 8, z, acc);
         c = run_end;
       } else {
-        // Rows at different rungs in this column: one pass per rung present.
-        for (int rr = jmin; rr <= jmax; ++rr) {
-          if (__any_sync(0xffffffffu, jr == rr) && jr == rr)
-            dispatch_cols<NB>(p.code[rr], rowbuf, pos, 1, tabs + p.slot[rr] * 512,
-                              xs + (c - cs) * 8, CF::ST * 8, z, acc);
+        // Rows at different rungs from column c on: for the rest of the stage,
+        // one pass per rung present, each lane running over its own columns
+        // at that rung (rungs rise along a row, so a lane's blocks are still
+        // taken in stream order).
+        int jhi = jr;
+        while (jhi < J - 1 && mybk[jhi] <= ce - 1) ++jhi;
+        jhi = __reduce_max_sync(0xffffffffu, jhi);
+        for (int rr = jmin; rr <= jhi; ++rr) {
+          const int ra = max(c, rr > 0 ? mybk[rr - 1] : 0);
+          const int rb = min(ce, rr < J - 1 ? mybk[rr] : nb);
+          const int cnt = rb > ra ? rb - ra : 0;
+          if (__any_sync(0xffffffffu, cnt > 0))
+            dispatch_cols<NB>(p.code[rr], rowbuf, pos, cnt, tabs + p.slot[rr] * 512,
+                              xs + (cnt > 0 ? ra - cs : 0) * 8, CF::ST * 8, z, acc);
         }
-        c += 1;
+        c = ce;
       }
       while (jr < J - 1 && nxt <= c) {
         ++jr;
@@ -437,8 +446,14 @@ static size_t smem_bytes() {
          sizeof(float) * Cfg<NB>::RG * kWarps * 32 * NB + 16;
 }
 
-// Cost-balanced ranges of the units of all tensors, one per CTA.
-static void partition(const seedq_layer *const *layers, int nt, MultiArgs &a) {
+// Cost-balanced ranges of the units of all tensors, one per CTA.  A group's
+// cost is its modeled time at batch n (block passes and the sum of k over
+// them); inside the group where a range is cut, the first row's rung profile,
+// scaled to the group's cost, places the cut.  One sweep over the groups
+// places all cuts in order.
+static void partition(const seedq_layer *const *layers, int nt, int n, MultiArgs &a) {
+  const double cb = cost_block(n);
+  auto gcost = [&](const seedq_layer *L, int64_t g) { return kCostK * L->h_gk[g] + cb * L->h_gp[g]; };
   int64_t U = 0;
   double total = 0.0;
   for (int i = 0; i < nt; ++i) {
@@ -446,7 +461,7 @@ static void partition(const seedq_layer *const *layers, int nt, MultiArgs &a) {
     const int64_t G = (L->args.R + 31) / 32;
     a.t[i].ubegin = U;
     U += G * L->args.nb;
-    total += L->h_gcost[G];
+    total += gcost(L, G);
   }
   int ctas = layers[0]->max_ctas;
   if (ctas > kMaxCtas) ctas = kMaxCtas;
@@ -454,41 +469,54 @@ static void partition(const seedq_layer *const *layers, int nt, MultiArgs &a) {
   a.ctas = ctas;
   a.cta_begin[0] = 0;
   a.cta_begin[ctas] = U;
-  int ti = 0;
-  double tbase = 0.0;  // cost of the tensors before ti
-  for (int c = 1; c < ctas; ++c) {
-    const double target = total * c / ctas;
+  int c = 1;
+  double tbase = 0.0;  // cost of the tensors before the current one
+  for (int ti = 0; ti < nt && c < ctas; ++ti) {
     const seedq_layer *L = layers[ti];
-    int64_t G = (L->args.R + 31) / 32;
-    while (ti + 1 < nt && tbase + L->h_gcost[G] <= target) {
-      tbase += L->h_gcost[G];
-      L = layers[++ti];
-      G = (L->args.R + 31) / 32;
-    }
-    const double lt = target - tbase;
-    int64_t lo = 0, hi = G - 1;  // last group with h_gcost[g] <= lt
-    while (lo < hi) {
-      const int64_t mid = (lo + hi + 1) / 2;
-      if (L->h_gcost[mid] <= lt) lo = mid;
-      else hi = mid - 1;
-    }
-    const int64_t g = lo;
+    const int64_t G = (L->args.R + 31) / 32;
     const int J = L->args.J, Jm1 = J > 1 ? J - 1 : 1, nb = L->args.nb;
-    const int32_t *b = L->h_repbk + g * Jm1;
-    double acc = L->h_gcost[g];
-    int col = nb, clo = 0;
-    for (int j = 0; j < J; ++j) {
-      const int chi = (j < J - 1) ? b[j] : nb;
-      const double seg = L->h_cost[j] * (chi - clo);
-      if (acc + seg > lt) {
-        col = clo + (int)((lt - acc) / L->h_cost[j]);
-        break;
+    for (int64_t g = 0; g < G && c < ctas; ++g) {
+      const double g0 = gcost(L, g), g1 = gcost(L, g + 1);
+      double target = total * c / ctas;
+      if (target - tbase >= g1) continue;
+      const int32_t *b = L->h_repbk + g * Jm1;
+      double rep = 0.0;
+      for (int j = 0, clo = 0; j < J; ++j) {
+        const int chi = (j < J - 1) ? b[j] : nb;
+        rep += (kCostK * L->k[j] + cb) * (chi - clo);
+        clo = chi;
       }
-      acc += seg;
-      clo = chi;
+      const double scale = rep > 0.0 ? (g1 - g0) / rep : 1.0;
+      while (c < ctas && target - tbase < g1) {
+        const double lt = target - tbase;
+        double acc = g0;
+        int col = nb, clo = 0;
+        for (int j = 0; j < J; ++j) {
+          const int chi = (j < J - 1) ? b[j] : nb;
+          const double per = (kCostK * L->k[j] + cb) * scale;
+          const double seg = per * (chi - clo);
+          if (acc + seg > lt) {
+            col = clo + (int)((lt - acc) / per);
+            break;
+          }
+          acc += seg;
+          clo = chi;
+        }
+        if (col < 0) col = 0;
+        if (col > nb) col = nb;
+        int64_t u = a.t[ti].ubegin + g * nb + col;
+        if (u <= a.cta_begin[c - 1]) u = a.cta_begin[c - 1] + 1;
+        if (u > U - (ctas - c)) u = U - (ctas - c);
+        a.cta_begin[c] = u;
+        ++c;
+        target = total * c / ctas;
+      }
     }
-    int64_t u = a.t[ti].ubegin + g * nb + col;
-    if (u <= a.cta_begin[c - 1]) u = a.cta_begin[c - 1] + 1;
+    tbase += gcost(L, G);
+  }
+  // Cuts left over by rounding at the very end of the sequence.
+  for (; c < ctas; ++c) {
+    int64_t u = a.cta_begin[c - 1] + 1;
     if (u > U - (ctas - c)) u = U - (ctas - c);
     a.cta_begin[c] = u;
   }
@@ -508,7 +536,7 @@ static seedq_status launch(const seedq_layer *const *layers, int nt, const uint1
     a->t[i].y = y[i];
     a->t[i].stream_bytes = layers[i]->stream_bytes;
   }
-  partition(layers, nt, *a);
+  partition(layers, nt, n, *a);
   static bool attr_set = false;
   seedq_status rc = SEEDQ_OK;
   if (!attr_set) {

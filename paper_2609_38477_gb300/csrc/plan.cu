@@ -310,29 +310,36 @@ static void free_layer(seedq_layer *L) {
   cudaFree(L->d_counters);
   cudaFree(L->d_slots);
   cudaFree(L->d_xperm);
-  free(L->h_gcost);
+  free(L->h_gp);
+  free(L->h_gk);
   free(L->h_repbk);
 
   free(L);
 }
 
 
-// Host-side cost profile of the tensor for the fused kernel's work partition.
-// Units are (row group, block) pairs in row-group-major order; a unit's cost is
-// modeled by the reconstruction work of its rung (8 (k+1) logic/FMA steps plus
-// a fixed per-block part), taken from the first row of the group in the
-// kernel's row order.  Kept: the cumulative cost per row group and those rows'
-// breakpoints, from which any cost target maps back to a (group, block) unit.
+// Host-side work profile of the tensor for the fused kernel's partition.
+// Units are (row group, block) pairs in row-group-major order.  The kernel
+// walks a row group's blocks in stages of a few columns; where all 32 rows of
+// the group sit at one rung it makes one pass per block, and from the first
+// column where they differ to the end of the stage it makes, for each rung
+// present, as many passes as the row with the most blocks at that rung in the
+// stage.  The profile counts those passes (stages aligned at block 0) and the
+// sum of k over them, per row group; the first row's breakpoints are kept to
+// place a cost target inside a group.
 static seedq_status build_costs(seedq_layer *L, cudaStream_t st) {
   const int64_t R = L->args.R;
-  const int J = L->args.J, Jm1 = J > 1 ? J - 1 : 1;
+  const int J = L->args.J, Jm1 = J > 1 ? J - 1 : 1, nb = L->args.nb;
   const int64_t G = (R + 31) / 32;
   int32_t *rowperm = (int32_t *)malloc(sizeof(int32_t) * R);
   int32_t *brk = (int32_t *)malloc(sizeof(int32_t) * R * Jm1);
-  L->h_gcost = (double *)malloc(sizeof(double) * (G + 1));
+  L->h_gp = (double *)malloc(sizeof(double) * (G + 1));
+  L->h_gk = (double *)malloc(sizeof(double) * (G + 1));
   L->h_repbk = (int32_t *)malloc(sizeof(int32_t) * G * Jm1);
+  const int nst = (nb + kCostStage - 1) / kCostStage;
+  uint8_t *mixed = (uint8_t *)malloc(nst);
   seedq_status rc = SEEDQ_OK;
-  if (!rowperm || !brk || !L->h_gcost || !L->h_repbk) rc = SEEDQ_ERR_NOMEM;
+  if (!rowperm || !brk || !L->h_gp || !L->h_gk || !L->h_repbk || !mixed) rc = SEEDQ_ERR_NOMEM;
   cudaError_t e = cudaSuccess;
   if (rc == SEEDQ_OK) e = cudaMemcpyAsync(rowperm, L->d_rowperm, sizeof(int32_t) * R, cudaMemcpyDeviceToHost, st);
   if (rc == SEEDQ_OK && e == cudaSuccess && J > 1)
@@ -340,22 +347,62 @@ static seedq_status build_costs(seedq_layer *L, cudaStream_t st) {
   if (rc == SEEDQ_OK && e == cudaSuccess) e = cudaStreamSynchronize(st);
   if (e != cudaSuccess) rc = cuda_fail(e);
   if (rc == SEEDQ_OK) {
-    for (int j = 0; j < J; ++j) L->h_cost[j] = 8.0 * (L->k[j] + 1) + 40.0;
-    L->h_gcost[0] = 0.0;
+    L->h_gp[0] = 0.0;
+    L->h_gk[0] = 0.0;
+    const int32_t *rowb[32];
     for (int64_t g = 0; g < G; ++g) {
-      const int32_t *b = brk + (int64_t)rowperm[g * 32] * Jm1;
+      int nr = 0;
+      for (int i = 0; i < 32 && g * 32 + i < R; ++i) rowb[nr++] = brk + (int64_t)rowperm[g * 32 + i] * Jm1;
+      const int32_t *b0 = rowb[0];
       int32_t *rb = L->h_repbk + g * Jm1;
-      double c = 0.0;
+      // The first row's profile.
+      double P = nb, K = 0.0;
       int lo = 0;
       for (int j = 0; j < J; ++j) {
-        const int hi = (j < J - 1) ? b[j] : L->args.nb;
-        if (j < J - 1) rb[j] = b[j];
-        c += L->h_cost[j] * (hi - lo);
+        const int hi = (j < J - 1) ? b0[j] : nb;
+        if (j < J - 1) rb[j] = b0[j];
+        K += (double)L->k[j] * (hi - lo);
         lo = hi;
       }
-      L->h_gcost[g + 1] = L->h_gcost[g] + c;
+      // Stages where the rows' breakpoints differ: replace the first row's
+      // passes there by the per-rung maxima over the rows.
+      bool any = false;
+      for (int s = 0; s < nst; ++s) mixed[s] = 0;
+      for (int j = 0; j < J - 1; ++j) {
+        int mn = b0[j], mx = b0[j];
+        for (int i = 1; i < nr; ++i) {
+          mn = rowb[i][j] < mn ? rowb[i][j] : mn;
+          mx = rowb[i][j] > mx ? rowb[i][j] : mx;
+        }
+        if (mn < mx) {
+          any = true;
+          const int s0 = mn / kCostStage, s1 = (mx - 1) / kCostStage;
+          for (int s = s0; s <= s1 && s < nst; ++s) mixed[s] = 1;
+        }
+      }
+      if (any) {
+        for (int s = 0; s < nst; ++s) {
+          if (!mixed[s]) continue;
+          const int cs = s * kCostStage, ce = (cs + kCostStage < nb) ? cs + kCostStage : nb;
+          for (int j = 0; j < J; ++j) {
+            int mxc = 0, c0 = 0;
+            for (int i = 0; i < nr; ++i) {
+              const int a = (j > 0) ? rowb[i][j - 1] : 0, z = (j < J - 1) ? rowb[i][j] : nb;
+              const int ra = a > cs ? a : cs, rz = z < ce ? z : ce;
+              const int cnt = rz > ra ? rz - ra : 0;
+              if (i == 0) c0 = cnt;
+              mxc = cnt > mxc ? cnt : mxc;
+            }
+            P += mxc - c0;
+            K += (double)L->k[j] * (mxc - c0);
+          }
+        }
+      }
+      L->h_gp[g + 1] = L->h_gp[g] + P;
+      L->h_gk[g + 1] = L->h_gk[g] + K;
     }
   }
+  free(mixed);
   free(rowperm);
   free(brk);
   return rc;

@@ -57,6 +57,19 @@ struct LayerArgs {
 
 }  // namespace seedq
 
+namespace seedq {
+// Modeled time of one block pass of the fused kernel at rung k with n
+// activation columns, in units of one coefficient: k + cost_block(n).  The
+// constants are fitted to the kernel's measured time per block on
+// single-rung tensors (S = 8..16, k = 2..6; n = 1, 4, 16; 2 and 8 between).
+constexpr double kCostK = 1.0;
+inline double cost_block(int n) {
+  return n <= 1 ? 3.7 : n <= 2 ? 5.3 : n <= 4 ? 8.4 : n <= 8 ? 12.5 : 19.6;
+}
+// Stage width (blocks) the work profile assumes.
+constexpr int kCostStage = 24;
+}  // namespace seedq
+
 struct seedq_layer {
   seedq::LayerArgs args;
   int32_t S[seedq::kMaxJ], k[seedq::kMaxJ];
@@ -80,9 +93,10 @@ struct seedq_layer {
   float *d_slots;
   float *d_xperm;
   int32_t max_ctas;      // CTAs of the fused kernel (one per SM)
-  double *h_gcost;       // host: cumulative modeled cost per row group (G + 1)
+  // Host-side work profile of the fused kernel, per row group (G + 1 entries,
+  // cumulative): block passes the warp makes, and the sum of k over them.
+  double *h_gp, *h_gk;
   int32_t *h_repbk;      // host: breakpoints of each row group's first row (G x (J-1))
-  double h_cost[seedq::kMaxJ];  // modeled cost of one block per rung
   uint64_t *d_row_off;
   uint64_t *d_tables;
   uint32_t *d_flags;
