@@ -50,7 +50,7 @@ typedef enum {
   SEEDQ_ERR_UNSUPPORTED = 6   /* rung or shape outside what the kernels implement */
 } seedq_status;
 
-/* A rung g = (S, k) of the hull (Sec. 3.1 "We call g = (S,k) a rung").
+/* A rung g = (S, k) of the hull: seed width S and coefficient count k (Sec. 3.1).
  * Supported: S in {8, 10, 12, 14, 16}, k in {2, ..., 6}. */
 typedef struct {
   int32_t S;
@@ -79,7 +79,7 @@ typedef struct {
  *   a             host, C floats, finite and >= 0, not all zero: the input
  *                 second moments (Eq. gamma or Eq. prop).
  *   rho           host, R floats finite and > 0, or NULL for all ones
- *                 (output factor of Sec. 3.3 "Output side").
+ *                 (the output-side factor of Sec. 3.3).
  *   tie_count     T_t of Alg. 2: the first T_t tied blocks in row-major order
  *                 take the lower rung.
  *   n_outliers    0..16 FP16 outlier columns (Sec. 3.5, App. A.6).
@@ -102,7 +102,7 @@ typedef struct {
 typedef struct seedq_layer seedq_layer;
 
 /* Build the decoder plan of one tensor (Alg. 2 lines computing imp, the floor
- * and the ladder; App. A.7 "Agreement"): column permutation (stable ascending
+ * and the ladder; App. A.7 on encoder/decoder agreement): column permutation (stable ascending
  * sort of a), unit-mean block means and row factors in fp64 in a fixed order,
  * per-row rung breakpoints after the tie pass, per-row bit offsets.  Runs on
  * the device on `cuda_stream` and waits for it (one-time set-up).  Allocates
@@ -154,12 +154,16 @@ seedq_status seedq_gemv(const seedq_layer *layer, const uint16_t *x, float *y,
 seedq_status seedq_gemm_small_batch(const seedq_layer *layer, const uint16_t *X,
                                     int32_t n, float *Y, void *cuda_stream);
 
-/* Several tensors in one launch (Alg. 2: tensors are decoded "in any order",
- * so the tensors of a decode step are independent): for i < count,
+/* Several tensors in one launch (Alg. 2 decodes each tensor on its own, in
+ * no fixed order, so the tensors of a decode step are independent): for i < count,
  * Y[i] = X[i] W_hat_i^T with X[i] device n x C_i bfloat16 and Y[i] device
  * n x R_i float32, as seedq_gemm_small_batch does for one layer.  count is
  * 1..8 and every layer must be bound and allow batch n.  Work is split across
- * the SMs by the modeled cost of all tensors together. */
+ * the SMs by the modeled cost of all tensors together.  The fused calls
+ * (gemv, gemm_small_batch, gemm_multi) use per-layer scratch (permuted
+ * activations, partial sums of row groups cut between SMs), so calls that
+ * involve the same layer must not run concurrently on different CUDA
+ * streams. */
 seedq_status seedq_gemm_multi(const seedq_layer *const *layers, int32_t count,
                               const uint16_t *const *X, int32_t n, float *const *Y,
                               void *cuda_stream);

@@ -1,7 +1,7 @@
 /*
  * Seed-Q oracle, side-information-free rung schedule (Sec. 3.3 Eq. imp and
- * the floor, Sec. 3.4 hull and Eq. ladder, App. A.5 ties, App. A.7
- * "Agreement", Alg. 1 allocation steps, Alg. 2 schedule steps).
+ * the floor, Sec. 3.4 hull and Eq. ladder, App. A.5 ties, App. A.7 on
+ * encoder/decoder agreement, Alg. 1 allocation steps, Alg. 2 schedule steps).
  * TEST INFRASTRUCTURE ONLY: see seedq_oracle.h.
  */
 #include <math.h>

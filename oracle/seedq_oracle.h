@@ -73,9 +73,9 @@ typedef struct {
   double q;             /* importance floor */
 } or_schedule;
 
-/* Per-tensor factors of Eq. imp, built in the fixed fp64 order of App. A.7
- * ("Agreement"): perm = stable ascending sort of a (Sec. 3.3 "Block
- * importance"); abar[c] = mean of a over block c of the permuted columns,
+/* Per-tensor factors of Eq. imp, built in the fixed fp64 order that App. A.7
+ * requires for encoder/decoder agreement: perm = stable ascending sort of a
+ * (Sec. 3.3, block importance); abar[c] = mean of a over block c of the permuted columns,
  * summed in i order, divided by its mean over c (summed in ascending c);
  * rho[r] = rho_r divided by its mean over r (summed in ascending r), or 1. */
 typedef struct {

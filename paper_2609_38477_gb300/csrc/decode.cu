@@ -19,7 +19,7 @@ __device__ __forceinline__ void decode_block(const LayerArgs &p, uint64_t off,
 
 // One thread per block; reads l(g_b) bits at the block's offset (row offset +
 // closed form over the row's rung breakpoints), writes 8 weights through the
-// inverse permutation (Alg. 2: "apply the inverse column permutation").
+// inverse permutation (the scatter step of Alg. 2).
 __global__ void __launch_bounds__(256) k_decode(const __grid_constant__ LayerArgs p, int64_t row0, int64_t nrows, float *W) {
   const int64_t total = nrows * (int64_t)p.nb;
   for (int64_t b = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; b < total;

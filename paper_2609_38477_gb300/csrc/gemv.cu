@@ -1,7 +1,7 @@
 // Fused reconstruction x matrix-vector product: y = W_hat x, and the decode-batch
 // skinny GEMM Y = X W_hat^T (n <= 16), for one tensor or for several tensors
 // in one launch (the tensors of a decode step are independent: Alg. 2 decodes
-// them "in any order").  W_hat is never written to memory; HBM carries only
+// each tensor on its own, in no fixed order).  W_hat is never written to memory; HBM carries only
 // the compressed streams, the plan rows and x / y.
 //
 // Layout: a lane owns a row.  A warp takes 32 rows (a row group, in the plan's

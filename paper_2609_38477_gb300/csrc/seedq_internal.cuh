@@ -15,7 +15,7 @@ constexpr int kMaxCols = 65536;
 constexpr int kTableSlots = 5;   // jump tables for S = 8, 10, 12, 14, 16
 
 // Supported rungs: S in {8,10,12,14,16}, k in {2..6} (the paper's grid, Sec. 3.1,
-// at the even seed widths its Table "Rung grids" uses).
+// at the even seed widths of its rung-grid table).
 __host__ __device__ constexpr int rung_code(int S, int k) { return ((S - 8) / 2) * 5 + (k - 2); }
 constexpr int kNumCodes = 25;
 inline bool rung_supported(int S, int k) {

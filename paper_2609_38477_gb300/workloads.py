@@ -87,7 +87,7 @@ def to_f16_bits(v: np.ndarray) -> np.ndarray:
 
 
 # ---------------------------------------------------------------------------
-# Damage tables: Table "Rung grids" (App. B.3), excess loss e(g) in nats per
+# Damage tables: the rung-grid table of App. B.3, excess loss e(g) in nats per
 # token over FP16 on WikiText-2 test, indexed by rung (S, k).
 DAMAGE_LLAMA2_7B = {
     (8, 3): 1.8746, (10, 3): 0.5852, (12, 3): 0.2249, (14, 3): 0.1182,

@@ -30,7 +30,7 @@ def _table_grids():
 # ------------------------------------------------------------------ Eq. rate
 
 def test_rate_matches_table_grids():
-    """Eq. rate with m = e = 4 reproduces every rate column entry of Table 'Rung grids'."""
+    """Eq. rate with m = e = 4 reproduces every rate entry of the rung-grid table (App. B.3)."""
     for S, k, rate, _, _ in _table_grids():
         assert O.block_bits(S, k) / 8.0 == rate
 
@@ -91,7 +91,7 @@ def test_taps_primitive_by_gf2_order(S):
 
 @pytest.mark.parametrize("S", [8, 11, 16])
 def test_sequence_period(S):
-    """'all 2^S - 1 seeds' (Sec. 3.1): the output bit sequence repeats with
+    """Sec. 3.1 searches every nonzero seed, 2^S - 1 of them: the output bit sequence repeats with
     period exactly 2^S - 1 and no smaller divisor."""
     taps = O.find_taps(S)
     n = (1 << S) - 1
@@ -280,8 +280,9 @@ def _hull_brute(points):
 
 
 def test_hull_llama2_7b_worked_example():
-    """Lower convex hull of the Llama-2-7B column of Table 'Rung grids': eight
-    rungs with decreasing slopes (Sec. 3.4; 'four to eight rungs', App. B.3)."""
+    """Lower convex hull of the Llama-2-7B column of the rung-grid table: eight
+    rungs with decreasing slopes (Sec. 3.4; App. B.3 reports hulls of four to
+    eight rungs)."""
     d = W.DAMAGE_LLAMA2_7B
     rungs, es, slopes = O.hull_rungs(d, 4.0)
     assert rungs == [(8, 3), (10, 3), (12, 3), (14, 3), (16, 3), (14, 4), (16, 5), (16, 6)]
