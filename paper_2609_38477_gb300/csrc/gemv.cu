@@ -271,36 +271,48 @@ __device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t 
     int jr = 0;
     while (jr < J - 1 && mybk[jr] <= cs) ++jr;
     int nxt = (jr < J - 1) ? mybk[jr] : nb;
+    // Passes over the stage's columns, each one run of blocks per lane at one
+    // rung, all through a single call site (one inlined copy of the rung
+    // loops keeps the instruction working set small).  Where all rows sit at
+    // one rung a pass is a run of columns shared by the 32 lanes; from the
+    // first column where they differ to the end of the stage there is one
+    // pass per rung present, each lane running over its own columns at that
+    // rung (rungs rise along a row, so a lane's blocks stay in stream order).
     int c = cs;
-    while (c < ce) {
-      const int jmin = __reduce_min_sync(0xffffffffu, jr), jmax = __reduce_max_sync(0xffffffffu, jr);
-      if (jmin == jmax) {
-        const int run_end = min((int)__reduce_min_sync(0xffffffffu, (unsigned)nxt), ce);
-        dispatch_cols<NB>(p.code[jmin], rowbuf, pos, run_end - c, tabs + p.slot[jmin] * 512,
-                          xs + (c - cs) * 8, CF::ST * 8, z, acc);
-        c = run_end;
-      } else {
-        // Rows at different rungs from column c on: for the rest of the stage,
-        // one pass per rung present, each lane running over its own columns
-        // at that rung (rungs rise along a row, so a lane's blocks are still
-        // taken in stream order).
-        int jhi = jr;
-        while (jhi < J - 1 && mybk[jhi] <= ce - 1) ++jhi;
-        jhi = __reduce_max_sync(0xffffffffu, jhi);
-        for (int rr = jmin; rr <= jhi; ++rr) {
-          const int ra = max(c, rr > 0 ? mybk[rr - 1] : 0);
-          const int rb = min(ce, rr < J - 1 ? mybk[rr] : nb);
-          const int cnt = rb > ra ? rb - ra : 0;
-          if (__any_sync(0xffffffffu, cnt > 0))
-            dispatch_cols<NB>(p.code[rr], rowbuf, pos, cnt, tabs + p.slot[rr] * 512,
-                              xs + (cnt > 0 ? ra - cs : 0) * 8, CF::ST * 8, z, acc);
+    int rr = -1, jhi = 0;
+    while (true) {
+      int j, cnt, xo;
+      if (rr < 0) {
+        if (c >= ce) break;
+        const int jmin = __reduce_min_sync(0xffffffffu, jr), jmax = __reduce_max_sync(0xffffffffu, jr);
+        if (jmin == jmax) {
+          const int run_end = min((int)__reduce_min_sync(0xffffffffu, (unsigned)nxt), ce);
+          j = jmin;
+          cnt = run_end - c;
+          xo = c - cs;
+          c = run_end;
+          while (jr < J - 1 && nxt <= c) {
+            ++jr;
+            nxt = (jr < J - 1) ? mybk[jr] : nb;
+          }
+        } else {
+          jhi = jr;
+          while (jhi < J - 1 && mybk[jhi] <= ce - 1) ++jhi;
+          jhi = __reduce_max_sync(0xffffffffu, jhi);
+          rr = jmin;
+          continue;
         }
-        c = ce;
+      } else {
+        if (rr > jhi) break;
+        const int ra = max(c, rr > 0 ? mybk[rr - 1] : 0);
+        const int rb = min(ce, rr < J - 1 ? mybk[rr] : nb);
+        j = rr++;
+        cnt = rb > ra ? rb - ra : 0;
+        xo = cnt > 0 ? ra - cs : 0;
+        if (!__any_sync(0xffffffffu, cnt > 0)) continue;
       }
-      while (jr < J - 1 && nxt <= c) {
-        ++jr;
-        nxt = (jr < J - 1) ? mybk[jr] : nb;
-      }
+      dispatch_cols<NB>(p.code[j], rowbuf, pos, cnt, tabs + p.slot[j] * 512, xs + xo * 8,
+                        CF::ST * 8, z, acc);
     }
     __syncwarp();
   }
@@ -339,6 +351,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ Mu
     uint4 *dst = reinterpret_cast<uint4 *>(tabs);
     for (int i = threadIdx.x; i < kTableSlots * 256; i += kThreads) dst[i] = __ldg(src + i);
   }
+  // The permuted activations come from the pre-kernel launched just before.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int cta = blockIdx.x;
   const int64_t u0 = a.cta_begin[cta], u1 = a.cta_begin[cta + 1];
   int64_t u = u0;
@@ -351,7 +365,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ Mu
     const int64_t tend = (ti + 1 < a.nt) ? a.t[ti + 1].ubegin : a.cta_begin[a.ctas];
     const int64_t rend = min(u1, tend);
     // The next round: up to RG row groups of this tensor.
-    Piece pcs[CF::RG];
+    // (In shared memory: the stage issue indexes it by a runtime piece number.)
+    __shared__ Piece pcs[4];
+    static_assert(CF::RG <= 4, "round size");
     int np = 0, nst_total = 0;
     int64_t uu = u;
     while (uu < rend && np < CF::RG) {
@@ -359,7 +375,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ Mu
       const int64_t g = lu / p.nb;
       const int ca = (int)(lu - g * p.nb);
       const int cb = (int)min((int64_t)p.nb, ca + (rend - uu));
-      pcs[np] = Piece{g, ca, cb};
+      if (threadIdx.x == 0) pcs[np] = Piece{g, ca, cb};
       nst_total += (cb - ca + CF::ST - 1) / CF::ST;
       ++np;
       uu += cb - ca;
@@ -423,20 +439,32 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ Mu
 
 // Activations in permuted column order, zero at outlier columns (their
 // contribution is added exactly by the epilogue): xperm[b][p] = x_b[perm[p]].
-__global__ void k_xperm(const __grid_constant__ MultiArgs a) {
-  for (int ti = 0; ti < a.nt; ++ti) {
-    const TensorArgs &T = a.t[ti];
-    const LayerArgs &p = T.p;
-    const int64_t total = (int64_t)a.n * p.C;
-    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
-         t += (int64_t)gridDim.x * blockDim.x) {
-      const int64_t b = t / p.C;
-      const int pc = (int)(t - b * p.C);
-      const int col = __ldg(p.perm + pc);
-      bool outl = false;
-      for (int o = 0; o < p.n_out; ++o) outl |= (p.out_cols[o] == col);
-      p.xperm[t] = outl ? 0.f : bf16_to_f32(__ldg(T.x + b * p.C + col));
-    }
+// One grid row per tensor.
+struct XpermArgs {
+  struct {
+    const int32_t *perm;
+    const uint16_t *x;
+    float *xperm;
+    int64_t C;
+    int32_t n_out;
+    int32_t out_cols[kMaxOutliers];
+  } t[kMaxTensors];
+  int n;
+};
+
+__global__ void k_xperm(const __grid_constant__ XpermArgs a) {
+  // The fused kernel may start launching now; it waits for this grid's writes.
+  asm volatile("griddepcontrol.launch_dependents;");
+  const auto &T = a.t[blockIdx.y];
+  const int64_t total = (int64_t)a.n * T.C;
+  for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
+       t += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t b = t / T.C;
+    const int pc = (int)(t - b * T.C);
+    const int col = __ldg(T.perm + pc);
+    bool outl = false;
+    for (int o = 0; o < T.n_out; ++o) outl |= (T.out_cols[o] == col);
+    T.xperm[t] = outl ? 0.f : bf16_to_f32(__ldg(T.x + b * T.C + col));
   }
 }
 
@@ -546,15 +574,38 @@ static seedq_status launch(const seedq_layer *const *layers, int nt, const uint1
     else attr_set = true;
   }
   if (rc == SEEDQ_OK) {
-    int64_t total = 0;
-    for (int i = 0; i < nt; ++i) total += (int64_t)n * layers[i]->args.C;
-    const int64_t want = (total + 255) / 256;
-    const int g = (int)(want < (int64_t)layers[0]->max_ctas * 8 ? want : (int64_t)layers[0]->max_ctas * 8);
-    k_xperm<<<g, 256, 0, st>>>(*a);
+    XpermArgs xa;
+    xa.n = n;
+    int64_t maxC = 0;
+    for (int i = 0; i < nt; ++i) {
+      const LayerArgs &p = layers[i]->args;
+      xa.t[i].perm = p.perm;
+      xa.t[i].x = x[i];
+      xa.t[i].xperm = p.xperm;
+      xa.t[i].C = p.C;
+      xa.t[i].n_out = p.n_out;
+      for (int o = 0; o < kMaxOutliers; ++o) xa.t[i].out_cols[o] = p.out_cols[o];
+      if (p.C > maxC) maxC = p.C;
+    }
+    const int64_t want = ((int64_t)n * maxC + 255) / 256;
+    const int gx = (int)(want < 64 ? want : 64);
+    k_xperm<<<dim3(gx, nt), 256, 0, st>>>(xa);
     cudaError_t e = cudaGetLastError();
     if (e == cudaSuccess) {
-      k_gemv<NB><<<a->ctas, kThreads, smem_bytes<NB>(), st>>>(*a);
-      e = cudaGetLastError();
+      // Programmatic dependent launch: the fused kernel's CTAs may start (and
+      // stage their jump tables) while the pre-kernel finishes; they wait for
+      // its writes before the first activation load.
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3(a->ctas);
+      cfg.blockDim = dim3(kThreads);
+      cfg.dynamicSmemBytes = smem_bytes<NB>();
+      cfg.stream = st;
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+      attr[0].val.programmaticStreamSerializationAllowed = 1;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      e = cudaLaunchKernelEx(&cfg, k_gemv<NB>, *a);
     }
     if (e != cudaSuccess) rc = cuda_fail(e);
   }
