@@ -31,7 +31,7 @@ FLUSH_BYTES = 512 << 20  # > 129 MB L2: written between timed steps
 def parse():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=400)
+    p.add_argument("--steps", type=int, default=2000)
     p.add_argument("--warmup", type=int, default=10)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default="c1")
@@ -74,8 +74,13 @@ class Clocks:
             os.close(fd)
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", self.index, f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "100"],
                 stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            # nvidia-smi takes a moment to start: wait for its first sample so
+            # the samples cover the timed region that follows.
+            t0 = time.time()
+            while time.time() - t0 < 5.0 and os.path.getsize(self.path) == 0:
+                time.sleep(0.02)
         except Exception:
             self.proc = None
 
@@ -258,7 +263,7 @@ def reference_arm(args):
     n = args.batch
     cores = cpu_cores()
     total_steps = args.steps + args.warmup
-    per_step = max(0.5, min(6.0, 150.0 / max(total_steps, 1)))
+    per_step = max(0.02, min(6.0, 150.0 / max(total_steps, 1)))
     run, frac, desc = oracle_sample(w, sched, n, per_step, cores)
     for _ in range(args.warmup):
         run()
@@ -333,6 +338,7 @@ def our_arm(args):
         step()
         b.record(stream)
     torch.cuda.synchronize()
+    clk = clocks.stop()
     dist_barrier()
     step_ms = [a.elapsed_time(b) for a, b in ev]
     # Per-tensor calls, for a per-tensor view of the same kernel (not the step).
@@ -347,7 +353,6 @@ def our_arm(args):
         torch.cuda.synchronize()
         for i in range(len(gts)):
             per_call[i].append(evs[i].elapsed_time(evs[i + 1]))
-    clk = clocks.stop()
 
     # End to end through the C ABI with host buffers: H2D of x, D2H of y.
     xh = [x.cpu().pin_memory() for x in xs]
