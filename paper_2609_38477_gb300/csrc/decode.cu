@@ -5,14 +5,14 @@
 
 namespace seedq {
 
-template <int S, int K>
-__device__ __forceinline__ void decode_block(const LayerArgs &p, uint64_t off,
+template <int K>
+__device__ __forceinline__ void decode_block(const LayerArgs &p, int S, uint64_t off,
                                              const uint64_t *tab, float *Wrow, int c) {
   uint32_t lo, hi;
-  load_bits<RungT<S, K>::NWORDS>(p.stream, off, lo, hi);
+  load_bits<3>(p.stream, off, lo, hi);  // the stream buffer ends in 16 bytes of slack
   float I[8], scale;
-  const RungConsts<S, K> rc(p.zero);
-  reconstruct<S, K>(lo, hi, tab, rc, I, scale);
+  const RungRt<K> rc(S, p.zero);
+  reconstruct_rt<K>(lo, hi, tab, rc, I, scale);
 #pragma unroll
   for (int i = 0; i < 8; ++i) Wrow[__ldg(p.perm + 8 * c + i)] = I[i] * scale;  // exact
 }
@@ -33,15 +33,14 @@ __global__ void __launch_bounds__(256) k_decode(const __grid_constant__ LayerArg
     const uint64_t off = __ldg(p.row_off + r) + bits_before(bk, p.J, p.L, p.nb, c);
     const uint64_t *tab = p.tables + (size_t)p.slot[g] * 512;
     float *Wrow = W + i * p.C;
-    switch (p.code[g]) {
-#define SEEDQ_CASE(S_, K_)                            \
-  case rung_code(S_, K_):                             \
-    decode_block<S_, K_>(p, off, tab, Wrow, c);       \
-    break;
-      SEEDQ_FOR_EACH_RUNG(SEEDQ_CASE)
-#undef SEEDQ_CASE
-      default:
-        atomicOr(p.flags, 1u);
+    const int S = rung_S(p.code[g]);
+    switch (rung_K(p.code[g])) {
+      case 2: decode_block<2>(p, S, off, tab, Wrow, c); break;
+      case 3: decode_block<3>(p, S, off, tab, Wrow, c); break;
+      case 4: decode_block<4>(p, S, off, tab, Wrow, c); break;
+      case 5: decode_block<5>(p, S, off, tab, Wrow, c); break;
+      case 6: decode_block<6>(p, S, off, tab, Wrow, c); break;
+      default: atomicOr(p.flags, 1u);
     }
   }
 }

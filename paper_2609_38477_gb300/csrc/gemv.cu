@@ -36,7 +36,7 @@ struct Cfg {
   // Columns per stage and row groups per round, sized so 12 warps' double
   // buffers and the round's partial sums fit in shared memory.
   static constexpr int ST = NB == 1 ? 24 : NB == 2 ? 16 : NB <= 8 ? 8 : 4;
-  static constexpr int RG = NB <= 4 ? 4 : 1;
+  static constexpr int RG = NB == 1 ? 8 : NB <= 4 ? 4 : 1;
   // 16-byte pieces per staged row: ST blocks of at most 44 bits, the 96-bit
   // read-ahead of the last block, and up to 15 + 15 bytes of alignment.
   static constexpr int PIECES = (ST * 44 / 8 + 12 + 30 + 15) / 16 + 1;
@@ -45,7 +45,7 @@ struct Cfg {
   static constexpr int RW = (PIECES % 2) ? PIECES * 4 : PIECES * 4 + 4;
   static constexpr int STREAM_WORDS = 2 * 32 * RW;  // per warp, double-buffered
   static constexpr int XFLOATS = 2 * ST * 8 * NB;   // per warp, double-buffered
-  static constexpr int WARP_BYTES = STREAM_WORDS * 4 + XFLOATS * 4 + 2 * 32 * 8 * 4;
+  static constexpr int WARP_BYTES = STREAM_WORDS * 4 + XFLOATS * 4 + 2 * 32 * 8 * 2;
 };
 
 struct TensorArgs {
@@ -90,14 +90,14 @@ __device__ __forceinline__ int cta_of(const MultiArgs &a, int64_t u) {
   return lo;
 }
 
-template <int S, int K, int NB>
+template <int K, int NB>
 __device__ __forceinline__ void block_fma(const uint32_t (&w)[3], uint32_t sh, const uint64_t *tab,
-                                          const RungConsts<S, K> &rc, const float *xc,
+                                          const RungRt<K> &rc, const float *xc,
                                           int xstride, float (&acc)[NB]) {
   const uint32_t lo = __funnelshift_r(w[0], w[1], sh);
   const uint32_t hi = __funnelshift_r(w[1], w[2], sh);
   float I[8], scale;
-  reconstruct<S, K>(lo, hi, tab, rc, I, scale);
+  reconstruct_rt<K>(lo, hi, tab, rc, I, scale);
 #pragma unroll
   for (int b = 0; b < NB; ++b) {
     const float4 x0 = *reinterpret_cast<const float4 *>(xc + b * xstride);
@@ -113,15 +113,12 @@ __device__ __forceinline__ void block_fma(const uint32_t (&w)[3], uint32_t sh, c
   }
 }
 
-// n consecutive columns of this lane's row at rung (S,K): pos is the bit
-// position of the first block in the lane's staged row buffer (advanced by
-// n * l(g)); xc the staged activations of the first column.
-template <int S, int K, int NB>
-__device__ __forceinline__ void run_cols(const uint32_t *rowbuf, uint32_t &pos, int n,
+template <int K, int NB>
+__device__ __forceinline__ void run_cols(int S, const uint32_t *rowbuf, uint32_t &pos, int n,
                                          const uint64_t *tab, const float *xc, int xstride,
                                          uint32_t z, float (&acc)[NB]) {
-  constexpr int L = RungT<S, K>::L;
-  const RungConsts<S, K> rc(z);
+  const uint32_t L = (uint32_t)(S + 4 * K + 4);
+  const RungRt<K> rc(S, z);
   uint32_t w[3];
   {
     const uint32_t *q = rowbuf + (pos >> 5);
@@ -139,7 +136,7 @@ __device__ __forceinline__ void run_cols(const uint32_t *rowbuf, uint32_t &pos, 
       w[1] = q[1];
       w[2] = q[2];
     }
-    block_fma<S, K, NB>(cur, sh, tab, rc, xc + i * 8, xstride, acc);
+    block_fma<K, NB>(cur, sh, tab, rc, xc + i * 8, xstride, acc);
   }
 }
 
@@ -147,20 +144,18 @@ template <int NB>
 __device__ __forceinline__ void dispatch_cols(int code, const uint32_t *rowbuf, uint32_t &pos, int n,
                                               const uint64_t *tab, const float *xc, int xstride,
                                               uint32_t z, float (&acc)[NB]) {
-  switch (code) {
-#define SEEDQ_CASE(S_, K_)                                                   \
-  case rung_code(S_, K_):                                                    \
-    run_cols<S_, K_, NB>(rowbuf, pos, n, tab, xc, xstride, z, acc);          \
-    break;
-    SEEDQ_FOR_EACH_RUNG(SEEDQ_CASE)
-#undef SEEDQ_CASE
-    default:
-      break;
+  const int S = rung_S(code);
+  switch (rung_K(code)) {
+    case 2: run_cols<2, NB>(S, rowbuf, pos, n, tab, xc, xstride, z, acc); break;
+    case 3: run_cols<3, NB>(S, rowbuf, pos, n, tab, xc, xstride, z, acc); break;
+    case 4: run_cols<4, NB>(S, rowbuf, pos, n, tab, xc, xstride, z, acc); break;
+    case 5: run_cols<5, NB>(S, rowbuf, pos, n, tab, xc, xstride, z, acc); break;
+    default: run_cols<6, NB>(S, rowbuf, pos, n, tab, xc, xstride, z, acc); break;
   }
 }
 
 // Bits of the lane's row before block x (rung j spans [bk[j-1], bk[j])).
-__device__ __forceinline__ uint32_t lane_bits_before(const int32_t *bk, int J, const int32_t *L,
+__device__ __forceinline__ uint32_t lane_bits_before(const int16_t *bk, int J, const int32_t *L,
                                                      int nb, int x) {
   uint32_t s = 0;
   int lo = 0;
@@ -185,7 +180,7 @@ struct Piece {
 template <int NB>
 __device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t z,
                                            const uint64_t *tabs, uint32_t *sbuf, float *xbuf,
-                                           int32_t *bk, const Piece *pcs, int np, int nst_total,
+                                           int16_t *bk, const Piece *pcs, int np, int nst_total,
                                            float *comb, int warp, int lane) {
   using CF = Cfg<NB>;
   const LayerArgs &p = T.p;
@@ -208,7 +203,7 @@ __device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t 
     const int64_t ridx = r0 + lane;
     const int64_t row = __ldg(p.rowperm + (ridx < p.R ? ridx : r0));
     const uint64_t roff = __ldg(p.row_off + row);
-    int32_t *mybk = bk + (sb * 32 + lane) * 8;
+    int16_t *mybk = bk + (sb * 32 + lane) * 8;
     for (int j = 0; j < J - 1; ++j) mybk[j] = __ldg(p.brk + row * (J - 1) + j);
     const uint64_t bit_cs = roff + lane_bits_before(mybk, J, p.L, nb, cs);
     const uint64_t b_lo = (bit_cs >> 3) & ~(uint64_t)15;
@@ -223,12 +218,9 @@ __device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t 
       piece_of[0] = pi; cs_of[0] = cs; ce_of[0] = ce; pos0[0] = p0;
     }
     uint32_t *rows = sbuf + sb * 32 * CF::RW;
-    for (int i = 0; i < 16; ++i) {
-      const int r = 2 * i + (lane >> 4), pc = lane & 15;
-      const uint64_t blo = __shfl_sync(0xffffffffu, b_lo, r);
-      const int npr = __shfl_sync(0xffffffffu, npc, r);
-      if (pc < npr) cp_async16(rows + r * CF::RW + pc * 4, gstream + blo + 16 * pc);
-    }
+#pragma unroll
+    for (int pc = 0; pc < CF::PIECES; ++pc)
+      if (pc < npc) cp_async16(rows + lane * CF::RW + pc * 4, gstream + b_lo + 16 * pc);
     float *xs = xbuf + sb * CF::ST * 8 * NB;
     const int nq = (ce - cs) * 2;  // 16-byte pieces per batch column
     for (int t2 = lane; t2 < n * nq; t2 += 32) {
@@ -265,7 +257,7 @@ __device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t 
       for (int b = 0; b < NB; ++b) acc[b] = 0.f;
       acc_piece = pi;
     }
-    const int32_t *mybk = bk + (sb * 32 + lane) * 8;
+    const int16_t *mybk = bk + (sb * 32 + lane) * 8;
     const uint32_t *rowbuf = sbuf + sb * 32 * CF::RW + lane * CF::RW;
     const float *xs = xbuf + sb * CF::ST * 8 * NB;
     int jr = 0;
@@ -342,7 +334,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ Mu
   uint8_t *mine = wbase + warp * CF::WARP_BYTES;
   uint32_t *sbuf = reinterpret_cast<uint32_t *>(mine);
   float *xbuf = reinterpret_cast<float *>(mine + CF::STREAM_WORDS * 4);
-  int32_t *bk = reinterpret_cast<int32_t *>(mine + CF::STREAM_WORDS * 4 + CF::XFLOATS * 4);
+  int16_t *bk = reinterpret_cast<int16_t *>(mine + CF::STREAM_WORDS * 4 + CF::XFLOATS * 4);
   float *comb = reinterpret_cast<float *>(wbase + kWarps * CF::WARP_BYTES);  // RG x kWarps x 32 x NB
   int *flag = reinterpret_cast<int *>(comb + CF::RG * kWarps * 32 * NB);
   {
@@ -366,8 +358,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ Mu
     const int64_t rend = min(u1, tend);
     // The next round: up to RG row groups of this tensor.
     // (In shared memory: the stage issue indexes it by a runtime piece number.)
-    __shared__ Piece pcs[4];
-    static_assert(CF::RG <= 4, "round size");
+    __shared__ Piece pcs[8];
+    static_assert(CF::RG <= 8, "round size");
     int np = 0, nst_total = 0;
     int64_t uu = u;
     while (uu < rend && np < CF::RG) {

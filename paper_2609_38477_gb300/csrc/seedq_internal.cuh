@@ -22,12 +22,8 @@ inline bool rung_supported(int S, int k) {
   return S >= 8 && S <= 16 && (S % 2) == 0 && k >= 2 && k <= 6;
 }
 
-#define SEEDQ_FOR_EACH_RUNG(X)                                                 \
-  X(8, 2) X(8, 3) X(8, 4) X(8, 5) X(8, 6)                                      \
-  X(10, 2) X(10, 3) X(10, 4) X(10, 5) X(10, 6)                                 \
-  X(12, 2) X(12, 3) X(12, 4) X(12, 5) X(12, 6)                                 \
-  X(14, 2) X(14, 3) X(14, 4) X(14, 5) X(14, 6)                                 \
-  X(16, 2) X(16, 3) X(16, 4) X(16, 5) X(16, 6)
+__host__ __device__ constexpr int rung_S(int code) { return 8 + 2 * (code / 5); }
+__host__ __device__ constexpr int rung_K(int code) { return 2 + code % 5; }
 
 // Everything a kernel needs about one layer, passed by value.
 struct LayerArgs {
@@ -52,7 +48,7 @@ struct LayerArgs {
   int32_t nslots;
   int32_t n_out;
   int32_t out_cols[kMaxOutliers];
-  uint32_t zero;            // 0; see RungConsts
+  uint32_t zero;            // 0; see RungRt
 };
 
 }  // namespace seedq
@@ -152,13 +148,6 @@ __device__ __forceinline__ void load_bits(const uint32_t *__restrict__ w, uint64
   hi = __funnelshift_r(w1, w2, sh);
 }
 
-template <int S, int K>
-struct RungT {
-  static constexpr int L = S + 4 * K + 4;
-  // Words touched by a block starting at any bit offset within a word.
-  static constexpr int NWORDS = (31 + L > 64) ? 3 : 2;
-};
-
 // ---------------------------------------------------------- reconstruction
 //
 // Eq. codec for one block, exactly: I[i] = sum_j t_j (x_{iK+j} - 2^{S-1}) as an
@@ -166,16 +155,22 @@ struct RungT {
 //
 // LFSR: the 64-bit sequence prefix Q = o_0..o_63 comes from two GF(2)-linear
 // jump tables indexed by the seed's bytes: tab[v] = Q(v), tab[256+v] =
-// Q((v mod 2^(S-8)) << 8), so the raw second byte of the field word indexes it.
+// Q((v mod 2^(S-8)) << 8), so the raw second byte of the field word indexes it
+// (for S = 8 the second half is all zero).
 //
-// States as floats: a state x_n sits at bits [n, n+S) of Q.  One funnel shift
-// brings a window of Q such that x_n lies at mantissa bits [23-S-d, 23-d) of a
-// 32-bit word; masking it and OR-ing exponent 127+S+d gives the float
-// 2^(S+d) + x_n.  A group of G consecutive states of one weight shares one
-// window (d = 0..G-1).  An FMA chain from init = -sum_j t_j (2^(S+d_j) + 2^(S-1))
-// then yields I exactly, provided every partial sum stays an integer below
-// 2^24 in magnitude; group_size() picks the largest G for which the worst case
-// (all |t_j| = 8) satisfies that.
+// Fields: f = bits [S, S+32) of the block puts E at [0, 4) and t_j at
+// [4+4j, 8+4j); a 4-bit field read under a fixed exponent gives t_j as a float.
+//
+// States as floats: Q is shifted left by 23 - S into three words (q2:q1:q0),
+// so state x_n sits at bits [23-S, 23) of the 32-bit window starting at bit n
+// (a compile-time position); state n-d of the same window lies at
+// [23-S-d, 23-d), and masking it and OR-ing exponent 127+S+d gives the float
+// 2^(S+d) + x_{n-d}.  A group of G consecutive states of one weight shares one
+// window.  An FMA chain from init = -sum_j t_j (2^(S+d_j) + 2^(S-1)) then
+// yields I exactly, provided every partial sum stays an integer below 2^24 in
+// magnitude; group_size() picks the largest G for which the worst case (all
+// |t_j| = 8) satisfies that, and the kernels use the value for S = 16, which
+// bounds every smaller width.  S is a run-time value: one code body per K.
 
 __host__ __device__ constexpr long long exact_bound(int S, int K, int G) {
   long long s = 0;
@@ -193,38 +188,6 @@ __host__ __device__ constexpr int group_size(int S, int K) {
   return g;
 }
 
-// Window (lo, mid, hi hold bits [0,32), [16,48), [32,64) of the block's field
-// word) and in-window bit position of the signed 4-bit field at absolute bit P;
-// the field must lie in mantissa bits [0, 23) of its window.
-__host__ __device__ constexpr int field_window(int P) { return P + 4 <= 23 ? 0 : P - 16 + 4 <= 23 ? 1 : 2; }
-__host__ __device__ constexpr int field_pos(int P) { return P - 16 * field_window(P); }
-
-// Per-rung constants kept in registers.  They are built from a runtime zero so
-// the compiler cannot fold them into instruction immediates: a LOP3 takes one
-// immediate at most, and (w & mask) | exponent must stay a single LOP3.
-template <int S, int K>
-struct RungConsts {
-  static constexpr int G = group_size(S, K);
-  uint32_t e_msk, e_x;           // shared exponent field
-  uint32_t t_msk[K], t_x[K];     // mantissa fields t_j
-  uint32_t s_msk[G], s_exp[G];   // state windows, by offset d within a group
-  __device__ __forceinline__ explicit RungConsts(uint32_t z) {
-    e_msk = (15u << S) ^ z;
-    e_x = (8u << S) ^ z;
-#pragma unroll
-    for (int j = 0; j < K; ++j) {
-      const int P = field_pos(S + 4 + 4 * j);
-      t_msk[j] = (15u << P) ^ z;
-      t_x[j] = ((8u << P) | ((uint32_t)(150 - P) << 23)) ^ z;
-    }
-#pragma unroll
-    for (int d = 0; d < G; ++d) {
-      s_msk[d] = (((1u << S) - 1u) << (23 - S - d)) ^ z;
-      s_exp[d] = ((uint32_t)(127 + S + d) << 23) ^ z;
-    }
-  }
-};
-
 // Single three-input logic instructions (the compiler otherwise splits them).
 __device__ __forceinline__ uint32_t lop_and_xor(uint32_t a, uint32_t m, uint32_t x) {
   uint32_t r;
@@ -237,82 +200,104 @@ __device__ __forceinline__ uint32_t lop_and_or(uint32_t a, uint32_t m, uint32_t 
   return r;
 }
 
-template <int S, int K, int J = 0>
-__device__ __forceinline__ void coeffs(uint32_t lo, uint32_t mid, uint32_t hi,
-                                       const RungConsts<S, K> &rc, float (&tf)[K]) {
-  if constexpr (J < K) {
-    constexpr int P = S + 4 + 4 * J;
-    constexpr int W = field_window(P);
-    constexpr int PP = field_pos(P);
-    static_assert(PP >= 0 && PP + 4 <= 23, "field outside the mantissa");
-    const uint32_t w = (W == 0) ? lo : (W == 1) ? mid : hi;
-    // Under exponent 150-PP the field reads as 2^(23-PP) + (t ^ 8) = 2^(23-PP) + 8 + t.
-    tf[J] = __uint_as_float(lop_and_xor(w, rc.t_msk[J], rc.t_x[J])) - (float)((1 << (23 - PP)) + 8);
-    coeffs<S, K, J + 1>(lo, mid, hi, rc, tf);
+// Per-rung constants kept in registers, built once per run of blocks.  They
+// are derived from a runtime zero so the compiler cannot fold them into
+// instruction immediates: a LOP3 takes one immediate at most, and
+// (w & mask) | exponent must stay a single LOP3.
+template <int K>
+struct RungRt {
+  static constexpr int G = group_size(16, K);
+  static_assert(exact_bound(16, K, G) < (1ll << 24), "FMA chain would round");
+  uint32_t S, qs;                 // seed width, 23 - S
+  uint32_t e_msk, e_x, sc;        // E field (at bit 0) and the scale's exponent offset
+  uint32_t t_msk[K], t_x[K];      // t_j fields
+  uint32_t s_msk[G], s_exp[G];    // state windows by offset d within a group
+  float cinit[K];                 // -(2^(S+d_j) + 2^(S-1))
+  __device__ __forceinline__ RungRt(int S_, uint32_t z) {
+    S = (uint32_t)S_;
+    qs = (uint32_t)(23 - S_);
+    e_msk = 15u ^ z;
+    e_x = 8u ^ z;
+    sc = ((uint32_t)(120 - S_) << 23) ^ z;
+#pragma unroll
+    for (int j = 0; j < K; ++j) {
+      const int P = (4 + 4 * j <= 19) ? 4 + 4 * j : 4 + 4 * j - 16;
+      t_msk[j] = (15u << P) ^ z;
+      t_x[j] = ((8u << P) | ((uint32_t)(150 - P) << 23)) ^ z;
+      const int d = (K - 1 - j) % G;
+      cinit[j] = -(float)((1 << (S_ + d)) + (1 << (S_ - 1)));
+    }
+#pragma unroll
+    for (int d = 0; d < G; ++d) {
+      s_msk[d] = ((((1u << S_) - 1u) << (23 - S_)) >> d) ^ z;
+      s_exp[d] = ((uint32_t)(127 + S_ + d) << 23) ^ z;
+    }
   }
+};
+
+// 32 bits of the 96-bit value (q2:q1:q0) starting at bit N (0 <= N < 64).
+template <int N>
+__device__ __forceinline__ uint32_t qwin3(uint32_t q0, uint32_t q1, uint32_t q2) {
+  if constexpr (N == 0) return q0;
+  else if constexpr (N < 32) return __funnelshift_r(q0, q1, N);
+  else if constexpr (N == 32) return q1;
+  else return __funnelshift_r(q1, q2, N - 32);
 }
 
-// 32 bits of Q (qlo | qhi << 32) starting at bit SH (SH may be negative: the
-// window then begins below bit 0 and its low bits are zero).
-template <int SH>
-__device__ __forceinline__ uint32_t qwin(uint32_t qlo, uint32_t qhi) {
-  if constexpr (SH <= -32) return 0u;
-  else if constexpr (SH < 0) return qlo << (-SH);
-  else if constexpr (SH == 0) return qlo;
-  else if constexpr (SH < 32) return __funnelshift_r(qlo, qhi, SH);
-  else if constexpr (SH == 32) return qhi;
-  else return qhi >> (SH - 32);
-}
-
-template <int S, int K, int G, int I, int J>
-__device__ __forceinline__ float state_chain(uint32_t qlo, uint32_t qhi, const RungConsts<S, K> &rc,
-                                             const float (&tf)[K], float acc) {
+template <int K, int I, int J>
+__device__ __forceinline__ float state_chain_rt(uint32_t q0, uint32_t q1, uint32_t q2,
+                                                const RungRt<K> &rc, const float (&tf)[K], float acc) {
   if constexpr (J < 0) {
     return acc;
   } else {
-    // Group holding state J of weight I: its top state jt sits at d = 0.
+    constexpr int G = RungRt<K>::G;
     constexpr int grp = (K - 1 - J) / G;
     constexpr int jt = K - 1 - grp * G;
     constexpr int d = jt - J;
-    const uint32_t win = qwin<I * K + jt + S - 23>(qlo, qhi);
+    const uint32_t win = qwin3<I * K + jt>(q0, q1, q2);
     acc = __fmaf_rn(tf[J], __uint_as_float(lop_and_or(win, rc.s_msk[d], rc.s_exp[d])), acc);
-    return state_chain<S, K, G, I, J - 1>(qlo, qhi, rc, tf, acc);
+    return state_chain_rt<K, I, J - 1>(q0, q1, q2, rc, tf, acc);
   }
 }
 
-template <int S, int K, int G, int I>
-__device__ __forceinline__ void weights_from(uint32_t qlo, uint32_t qhi, const RungConsts<S, K> &rc,
-                                             const float (&tf)[K], float init, float (&Iv)[8]) {
+template <int K, int I>
+__device__ __forceinline__ void weights_from_rt(uint32_t q0, uint32_t q1, uint32_t q2,
+                                                const RungRt<K> &rc, const float (&tf)[K],
+                                                float init, float (&Iv)[8]) {
   if constexpr (I < 8) {
-    Iv[I] = state_chain<S, K, G, I, K - 1>(qlo, qhi, rc, tf, init);
-    weights_from<S, K, G, I + 1>(qlo, qhi, rc, tf, init, Iv);
+    Iv[I] = state_chain_rt<K, I, K - 1>(q0, q1, q2, rc, tf, init);
+    weights_from_rt<K, I + 1>(q0, q1, q2, rc, tf, init, Iv);
   }
 }
 
 // lo, hi: the block's 64 field bits starting at its first bit.
-template <int S, int K>
-__device__ __forceinline__ void reconstruct(uint32_t lo, uint32_t hi, const uint64_t *tab,
-                                            const RungConsts<S, K> &rc, float (&I)[8],
-                                            float &scale) {
-  constexpr int G = RungConsts<S, K>::G;
-  static_assert(exact_bound(S, K, G) < (1ll << 24), "FMA chain would round");
-  uint64_t Q = tab[lo & 255u];
-  if (S > 8) Q ^= tab[256 + __byte_perm(lo, 0, 0x4441)];
+template <int K>
+__device__ __forceinline__ void reconstruct_rt(uint32_t lo, uint32_t hi, const uint64_t *tab,
+                                               const RungRt<K> &rc, float (&I)[8], float &scale) {
+  // For S = 8 the second table half is all zero, so both lookups are always valid.
+  const uint64_t Q = tab[lo & 255u] ^ tab[256 + __byte_perm(lo, 0, 0x4441)];
   const uint32_t qlo = (uint32_t)Q, qhi = (uint32_t)(Q >> 32);
-  // scale = 2^(E-S+1): (E+8) = field ^ 8 lands in the exponent via one multiply-add.
-  const uint32_t e8 = lop_and_xor(lo, rc.e_msk, rc.e_x);
-  scale = __uint_as_float(e8 * (1u << (23 - S)) + ((uint32_t)(127 - S + 1 - 8) << 23));
-  const uint32_t mid = __funnelshift_r(lo, hi, 16);
+  const uint32_t q0 = qlo << rc.qs;
+  const uint32_t q1 = __funnelshift_l(qlo, qhi, rc.qs);
+  const uint32_t q2 = __funnelshift_l(qhi, 0u, rc.qs);
+  const uint32_t f = __funnelshift_r(lo, hi, rc.S);
+  const uint32_t e8 = lop_and_xor(f, rc.e_msk, rc.e_x);
+  scale = __uint_as_float(e8 * (1u << 23) + rc.sc);
   float tf[K];
-  coeffs<S, K>(lo, mid, hi, rc, tf);
-  float init = 0.f;
+  uint32_t f2 = 0;
+  if constexpr (K > 4) f2 = f >> 16;
 #pragma unroll
   for (int j = 0; j < K; ++j) {
-    const int d = (K - 1 - j) % G;
-    init = __fmaf_rn(tf[j], -(float)((1 << (S + d)) + (1 << (S - 1))), init);
+    const int P = (4 + 4 * j <= 19) ? 4 + 4 * j : 4 + 4 * j - 16;
+    const uint32_t w = (4 + 4 * j <= 19) ? f : f2;
+    tf[j] = __uint_as_float(lop_and_xor(w, rc.t_msk[j], rc.t_x[j])) - (float)((1 << (23 - P)) + 8);
   }
-  weights_from<S, K, G, 0>(qlo, qhi, rc, tf, init, I);
+  float init = 0.f;
+#pragma unroll
+  for (int j = 0; j < K; ++j) init = __fmaf_rn(tf[j], rc.cinit[j], init);
+  weights_from_rt<K, 0>(q0, q1, q2, rc, tf, init, I);
 }
+
 
 __host__ __device__ inline uint64_t stream_bytes_required(uint64_t bits) {
   return ((bits + 7) / 8 + 15) / 16 * 16 + 16;
