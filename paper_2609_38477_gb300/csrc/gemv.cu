@@ -90,18 +90,42 @@ __device__ __forceinline__ int cta_of(const MultiArgs &a, int64_t u) {
   return lo;
 }
 
+// Packed pair of fp32 values (lane-wise fma.rn.f32x2 on sm_100 and later).
+__device__ __forceinline__ uint64_t pk2(float a, float b) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+  return r;
+}
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t mul2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
+// One block: reconstruct its 8 weights and add scale * sum_i I_i x_b[i] to
+// acc[b].  xc holds the block's activations weight-major, NB per weight
+// (xc[i * NB + b]).  Per batch column the products form two chains (weights
+// 0-3 and 4-7); at NB >= 2 two batch columns share each packed instruction.
 template <int K, int NB>
 __device__ __forceinline__ void block_fma(const uint32_t (&w)[3], uint32_t sh, const uint64_t *tab,
-                                          const RungRt<K> &rc, const float *xc,
-                                          int xstride, float (&acc)[NB]) {
+                                          const RungRt<K> &rc, const float *xc, float (&acc)[NB]) {
   const uint32_t lo = __funnelshift_r(w[0], w[1], sh);
   const uint32_t hi = __funnelshift_r(w[1], w[2], sh);
   float I[8], scale;
   reconstruct_rt<K>(lo, hi, tab, rc, I, scale);
-#pragma unroll
-  for (int b = 0; b < NB; ++b) {
-    const float4 x0 = *reinterpret_cast<const float4 *>(xc + b * xstride);
-    const float4 x1 = *reinterpret_cast<const float4 *>(xc + b * xstride + 4);
+  if constexpr (NB == 1) {
+    const float4 x0 = *reinterpret_cast<const float4 *>(xc);
+    const float4 x1 = *reinterpret_cast<const float4 *>(xc + 4);
     float s0 = I[0] * x0.x, s1 = I[4] * x1.x;
     s0 = __fmaf_rn(I[1], x0.y, s0);
     s1 = __fmaf_rn(I[5], x1.y, s1);
@@ -109,13 +133,32 @@ __device__ __forceinline__ void block_fma(const uint32_t (&w)[3], uint32_t sh, c
     s1 = __fmaf_rn(I[6], x1.z, s1);
     s0 = __fmaf_rn(I[3], x0.w, s0);
     s1 = __fmaf_rn(I[7], x1.w, s1);
-    acc[b] = __fmaf_rn(scale, s0 + s1, acc[b]);
+    acc[0] = __fmaf_rn(scale, s0 + s1, acc[0]);
+  } else {
+    const uint64_t *x2 = reinterpret_cast<const uint64_t *>(xc);  // pairs of batch columns
+    uint64_t Ip[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) Ip[i] = pk2(I[i], I[i]);
+    const uint64_t sp = pk2(scale, scale);
+#pragma unroll
+    for (int q = 0; q < NB / 2; ++q) {
+      uint64_t s0 = mul2(Ip[0], x2[0 * (NB / 2) + q]), s1 = mul2(Ip[4], x2[4 * (NB / 2) + q]);
+      s0 = fma2(Ip[1], x2[1 * (NB / 2) + q], s0);
+      s1 = fma2(Ip[5], x2[5 * (NB / 2) + q], s1);
+      s0 = fma2(Ip[2], x2[2 * (NB / 2) + q], s0);
+      s1 = fma2(Ip[6], x2[6 * (NB / 2) + q], s1);
+      s0 = fma2(Ip[3], x2[3 * (NB / 2) + q], s0);
+      s1 = fma2(Ip[7], x2[7 * (NB / 2) + q], s1);
+      const uint64_t a = fma2(sp, add2(s0, s1), pk2(acc[2 * q], acc[2 * q + 1]));
+      acc[2 * q] = __uint_as_float((uint32_t)a);
+      acc[2 * q + 1] = __uint_as_float((uint32_t)(a >> 32));
+    }
   }
 }
 
 template <int K, int NB>
 __device__ __forceinline__ void run_cols(int S, const uint32_t *rowbuf, uint32_t &pos, int n,
-                                         const uint64_t *tab, const float *xc, int xstride,
+                                         const uint64_t *tab, const float *xc,
                                          uint32_t z, float (&acc)[NB]) {
   const uint32_t L = (uint32_t)(S + 4 * K + 4);
   const RungRt<K> rc(S, z);
@@ -136,21 +179,21 @@ __device__ __forceinline__ void run_cols(int S, const uint32_t *rowbuf, uint32_t
       w[1] = q[1];
       w[2] = q[2];
     }
-    block_fma<K, NB>(cur, sh, tab, rc, xc + i * 8, xstride, acc);
+    block_fma<K, NB>(cur, sh, tab, rc, xc + i * 8 * NB, acc);
   }
 }
 
 template <int NB>
 __device__ __forceinline__ void dispatch_cols(int code, const uint32_t *rowbuf, uint32_t &pos, int n,
-                                              const uint64_t *tab, const float *xc, int xstride,
+                                              const uint64_t *tab, const float *xc,
                                               uint32_t z, float (&acc)[NB]) {
   const int S = rung_S(code);
   switch (rung_K(code)) {
-    case 2: run_cols<2, NB>(S, rowbuf, pos, n, tab, xc, xstride, z, acc); break;
-    case 3: run_cols<3, NB>(S, rowbuf, pos, n, tab, xc, xstride, z, acc); break;
-    case 4: run_cols<4, NB>(S, rowbuf, pos, n, tab, xc, xstride, z, acc); break;
-    case 5: run_cols<5, NB>(S, rowbuf, pos, n, tab, xc, xstride, z, acc); break;
-    default: run_cols<6, NB>(S, rowbuf, pos, n, tab, xc, xstride, z, acc); break;
+    case 2: run_cols<2, NB>(S, rowbuf, pos, n, tab, xc, z, acc); break;
+    case 3: run_cols<3, NB>(S, rowbuf, pos, n, tab, xc, z, acc); break;
+    case 4: run_cols<4, NB>(S, rowbuf, pos, n, tab, xc, z, acc); break;
+    case 5: run_cols<5, NB>(S, rowbuf, pos, n, tab, xc, z, acc); break;
+    default: run_cols<6, NB>(S, rowbuf, pos, n, tab, xc, z, acc); break;
   }
 }
 
@@ -222,11 +265,11 @@ __device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t 
     for (int pc = 0; pc < CF::PIECES; ++pc)
       if (pc < npc) cp_async16(rows + lane * CF::RW + pc * 4, gstream + b_lo + 16 * pc);
     float *xs = xbuf + sb * CF::ST * 8 * NB;
-    const int nq = (ce - cs) * 2;  // 16-byte pieces per batch column
-    for (int t2 = lane; t2 < n * nq; t2 += 32) {
-      const int b = t2 / nq, q = t2 - b * nq;
-      cp_async16(xs + b * CF::ST * 8 + q * 4, p.xperm + (int64_t)b * p.C + cs * 8 + q * 4);
-    }
+    // Activations of the stage's columns: contiguous in the weight-major
+    // scratch layout (NB values per weight).
+    const int nq = (ce - cs) * 2 * NB;  // 16-byte pieces
+    for (int q = lane; q < nq; q += 32)
+      cp_async16(xs + q * 4, p.xperm + (int64_t)cs * 8 * NB + q * 4);
     cp_async_commit();
   };
 
@@ -303,8 +346,8 @@ __device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t 
         xo = cnt > 0 ? ra - cs : 0;
         if (!__any_sync(0xffffffffu, cnt > 0)) continue;
       }
-      dispatch_cols<NB>(p.code[j], rowbuf, pos, cnt, tabs + p.slot[j] * 512, xs + xo * 8,
-                        CF::ST * 8, z, acc);
+      dispatch_cols<NB>(p.code[j], rowbuf, pos, cnt, tabs + p.slot[j] * 512, xs + xo * 8 * NB,
+                        z, acc);
     }
     __syncwarp();
   }
@@ -430,8 +473,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ Mu
 }
 
 // Activations in permuted column order, zero at outlier columns (their
-// contribution is added exactly by the epilogue): xperm[b][p] = x_b[perm[p]].
-// One grid row per tensor.
+// contribution is added exactly by the epilogue), weight-major with NB values
+// per weight: xperm[p * NB + b] = x_b[perm[p]] (0 for b >= n).  One grid row
+// per tensor.
 struct XpermArgs {
   struct {
     const int32_t *perm;
@@ -441,22 +485,27 @@ struct XpermArgs {
     int32_t n_out;
     int32_t out_cols[kMaxOutliers];
   } t[kMaxTensors];
-  int n;
+  int n;   // batch columns
+  int nbt; // batch template: values per weight in the scratch layout
 };
 
 __global__ void k_xperm(const __grid_constant__ XpermArgs a) {
   // The fused kernel may start launching now; it waits for this grid's writes.
   asm volatile("griddepcontrol.launch_dependents;");
   const auto &T = a.t[blockIdx.y];
-  const int64_t total = (int64_t)a.n * T.C;
+  const int64_t total = (int64_t)a.nbt * T.C;
   for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
        t += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t b = t / T.C;
-    const int pc = (int)(t - b * T.C);
-    const int col = __ldg(T.perm + pc);
-    bool outl = false;
-    for (int o = 0; o < T.n_out; ++o) outl |= (T.out_cols[o] == col);
-    T.xperm[t] = outl ? 0.f : bf16_to_f32(__ldg(T.x + b * T.C + col));
+    const int64_t pc = t / a.nbt;
+    const int b = (int)(t - pc * a.nbt);
+    float v = 0.f;
+    if (b < a.n) {
+      const int col = __ldg(T.perm + pc);
+      bool outl = false;
+      for (int o = 0; o < T.n_out; ++o) outl |= (T.out_cols[o] == col);
+      v = outl ? 0.f : bf16_to_f32(__ldg(T.x + (int64_t)b * T.C + col));
+    }
+    T.xperm[t] = v;
   }
 }
 
@@ -568,6 +617,7 @@ static seedq_status launch(const seedq_layer *const *layers, int nt, const uint1
   if (rc == SEEDQ_OK) {
     XpermArgs xa;
     xa.n = n;
+    xa.nbt = NB;
     int64_t maxC = 0;
     for (int i = 0; i < nt; ++i) {
       const LayerArgs &p = layers[i]->args;
@@ -579,7 +629,7 @@ static seedq_status launch(const seedq_layer *const *layers, int nt, const uint1
       for (int o = 0; o < kMaxOutliers; ++o) xa.t[i].out_cols[o] = p.out_cols[o];
       if (p.C > maxC) maxC = p.C;
     }
-    const int64_t want = ((int64_t)n * maxC + 255) / 256;
+    const int64_t want = ((int64_t)NB * maxC + 255) / 256;
     const int gx = (int)(want < 64 ? want : 64);
     k_xperm<<<dim3(gx, nt), 256, 0, st>>>(xa);
     cudaError_t e = cudaGetLastError();

@@ -549,7 +549,9 @@ seedq_status seedq_layer_prepare(const seedq_layer_desc *d, const seedq_schedule
   ALLOC(L->d_rowperm, sizeof(int32_t) * R);
   ALLOC(L->d_counters, sizeof(int32_t) * ngroups);
   ALLOC(L->d_slots, sizeof(float) * L->max_ctas * 2 * 32 * kMaxBatch);
-  ALLOC(L->d_xperm, sizeof(float) * C * mb);
+  // Weight-major activations, padded to the kernel's batch template.
+  const int mbt = mb <= 1 ? 1 : mb <= 2 ? 2 : mb <= 4 ? 4 : mb <= 8 ? 8 : 16;
+  ALLOC(L->d_xperm, sizeof(float) * C * mbt);
 
 #undef ALLOC
   L->args.perm = L->d_perm;

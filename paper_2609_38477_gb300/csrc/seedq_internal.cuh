@@ -35,7 +35,7 @@ struct LayerArgs {
   const int32_t *invperm;   // C: position of column j in the permuted order
   const uint16_t *out_vals; // R x n_out binary16
   const int32_t *rowperm;   // R: order in which rows are grouped 32 to a warp
-  float *xperm;             // max_batch x C: activations in permuted column order
+  float *xperm;             // C x n: activations in permuted order, weight-major
   int32_t *counters;        // row groups: arrivals of partial sums (0 between calls)
   float *slots;             // max_ctas x 2 x 32 x 16 partial sums of row groups
   uint32_t *flags;
