@@ -189,6 +189,45 @@ seedq_status seedq_last_device_error(const seedq_layer *layer, uint32_t *flags);
  * o_{t+i} feeds o_{t+S}); 0 for widths outside 8..16.  Host function. */
 uint32_t seedq_lfsr_taps(int32_t S);
 
+/* ---------------------------------------------------------------- encoder
+ * The exhaustive seed search of Eq. codec (Sec. 3.1: every seed of the S-bit
+ * LFSR, least-squares coefficients quantized to 4-bit mantissas under one
+ * 4-bit exponent, smallest quantized error), run per block at its rung as
+ * Alg. 1's emit step does, and the packing of the chosen fields into the
+ * stream layout above.  Per seed: U(s) as in Eq. codec; the k x k normal
+ * equations solved in fp64 by Gaussian elimination with partial pivoting
+ * (seeds with a pivot below 1e-12 are skipped); E = the smallest value in
+ * [-8, 7] for which every round-half-even t*_j 2^-E lies in [-8, 7] (7 if
+ * none); t_j those values clamped to [-8, 7]; error = sum_i (w_i - w_hat_i)^2
+ * in fp64.  The smallest error wins, ties to the smaller seed.  Every product
+ * and sum is rounded separately in a fixed order, so the choice is the same
+ * on any IEEE machine running these steps.
+ *
+ * Outputs per block b: seed[b] (uint32), E[b] (int8), t[6 b + j] (int8, j < k;
+ * the rest 0), err[b] (double; may be NULL).  All device pointers; work is
+ * enqueued on cuda_stream. */
+
+/* Blocks at one rung (S even in 8..16, k in 2..6): w is device nblocks x 8
+ * float32, row-major (one block per row).  Other rungs: SEEDQ_ERR_UNSUPPORTED. */
+seedq_status seedq_encode_blocks(int32_t S, int32_t k, const float *w, int64_t nblocks,
+                                 uint32_t *seed, int8_t *E, int8_t *t, double *err,
+                                 void *cuda_stream);
+
+/* Every block of a prepared layer at the rung its plan assigns: W is device
+ * R x C float32 in the original column order (block (r, c) holds the columns
+ * perm[8c .. 8c+7] of row r); outputs have R x (C/8) entries in row-major
+ * block order. */
+seedq_status seedq_encode_layer(const seedq_layer *layer, const float *W, uint32_t *seed,
+                                int8_t *E, int8_t *t, double *err, void *cuda_stream);
+
+/* Pack per-block fields (as seedq_encode_layer writes them) into a stream
+ * buffer: device, 16-byte aligned, stream_bytes >= seedq_stream_bytes_required
+ * (plan bits); zeroed first.  The result binds to the layer with
+ * seedq_layer_bind_stream. */
+seedq_status seedq_pack_stream(const seedq_layer *layer, const uint32_t *seed, const int8_t *E,
+                               const int8_t *t, void *stream, uint64_t stream_bytes,
+                               void *cuda_stream);
+
 /* Fill a stream buffer with the synthetic payload of the workload recipe:
  * block b of the tensor (row-major) draws h = splitmix64 output number b from
  * state `key` and uses seed = 1 + (h>>32) mod (2^S-1), E = -8 + ((h>>24)&255)

@@ -1,0 +1,347 @@
+// Encoder: the exhaustive seed search of Eq. codec (Sec. 3.1, run per block at
+// its rung by Alg. 1's emit step) and the packing of the resulting fields into
+// the stream layout the decoder reads.
+//
+// For every seed s in [1, 2^S - 1] the search forms U(s) (8 x k entries
+// (x_{ik+j} - 2^{S-1}) / 2^{S-1}), solves the k x k normal equations for the
+// least-squares coefficients by Gaussian elimination with partial pivoting,
+// picks the smallest shared exponent E in [-8, 7] whose round-half-even
+// mantissas t_j * 2^-E all lie in [-8, 7] (E = 7 when none does), and scores
+// the quantized block by its squared error.  The smallest error wins; ties go
+// to the smaller seed.  Seeds whose system has a pivot below 1e-12 are skipped.
+//
+// Arithmetic: fp64, each product and sum rounded separately (no contraction),
+// in the order written above, so every decision (the pivot row, the exponent,
+// the mantissas, the winning seed) is the same on any IEEE machine that runs
+// the same steps.  Three exact rescalings keep the work small without
+// changing any rounded value: U is kept as the integers x - 2^{S-1} (every
+// product and sum of the normal matrix is then an exact integer), and the
+// powers of two dropped from the matrix (2^{2-2S}) and right-hand side
+// (2^{1-S}) are restored exactly in the exponent arithmetic; Gaussian
+// elimination commutes with scaling by powers of two.
+//
+// Work split: one warp per block, lanes striding over the seeds, then a warp
+// reduction on (error, seed).
+#include "seedq_internal.cuh"
+
+namespace seedq {
+
+constexpr int kEncWarps = 8;
+
+// Power of two 2^e as a double (|e| well inside the normal range).
+__device__ __forceinline__ double pow2d(int e) { return __longlong_as_double((long long)(1023 + e) << 52); }
+
+// All k rounded mantissas of tstar * 2^-E lie in [-8, 7].
+template <int K>
+__device__ __forceinline__ bool fits(const double (&ts)[K], double scale) {
+  bool ok = true;
+#pragma unroll
+  for (int j = 0; j < K; ++j) {
+    const double m = rint(__dmul_rn(ts[j], scale));
+    ok = ok && (m >= -8.0) && (m <= 7.0);
+  }
+  return ok;
+}
+
+// Search all seeds of one block (w: 8 weights) for the lane's share of seeds.
+// Returns the lane's best (error, seed, E, t) in the order of the scan.
+template <int K>
+__device__ __forceinline__ void search_block(int S, const uint64_t *tab, const double (&w)[8], int lane,
+                                             double &best, uint32_t &bseed, int &bE, int (&bt)[6]) {
+  const uint32_t mask = (1u << S) - 1u;
+  const int h = 1 << (S - 1);
+  // Pivot threshold of the unscaled matrix: 1e-12 * 2^(2S-2), exact.
+  const double thr = __dmul_rn(1e-12, pow2d(2 * S - 2));
+  best = __longlong_as_double(0x7ff0000000000000ll);  // +inf
+  bseed = 0;
+  bE = 0;
+#pragma unroll
+  for (int j = 0; j < 6; ++j) bt[j] = 0;
+  const uint32_t nseeds = mask;  // seeds 1 .. 2^S - 1
+  for (uint32_t s = 1 + lane; s <= nseeds; s += 32) {
+    const uint64_t Q = tab[s & 255u] ^ tab[256 + ((s >> 8) & 255u)];
+    int u[8][K];
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+#pragma unroll
+      for (int j = 0; j < K; ++j) u[i][j] = (int)((uint32_t)(Q >> (i * K + j)) & mask) - h;
+    // Normal equations (unscaled): A[p][q] exact integers, b[p] rounded in i order.
+    double A[K][K], b[K];
+#pragma unroll
+    for (int p = 0; p < K; ++p) {
+      double r = 0.0;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) r = __dadd_rn(r, __dmul_rn((double)u[i][p], w[i]));
+      b[p] = r;
+#pragma unroll
+      for (int q = p; q < K; ++q) {
+        long long acc = 0;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) acc += (long long)(u[i][p] * u[i][q]);
+        A[p][q] = (double)acc;
+        A[q][p] = A[p][q];
+      }
+    }
+    // Gaussian elimination with partial pivoting (first row of largest |pivot|).
+    bool singular = false;
+#pragma unroll
+    for (int c = 0; c < K; ++c) {
+      int pr = c;
+      double pv = fabs(A[c][c]);
+#pragma unroll
+      for (int r = c + 1; r < K; ++r) {
+        const double v = fabs(A[r][c]);
+        if (v > pv) {
+          pv = v;
+          pr = r;
+        }
+      }
+      singular = singular || (pv < thr);
+#pragma unroll
+      for (int r = c + 1; r < K; ++r) {
+        if (pr == r) {
+#pragma unroll
+          for (int q = c; q < K; ++q) {
+            const double tmp = A[c][q];
+            A[c][q] = A[r][q];
+            A[r][q] = tmp;
+          }
+          const double tb = b[c];
+          b[c] = b[r];
+          b[r] = tb;
+        }
+      }
+#pragma unroll
+      for (int r = c + 1; r < K; ++r) {
+        const double f = A[r][c] / A[c][c];
+#pragma unroll
+        for (int q = c + 1; q < K; ++q) A[r][q] = __dsub_rn(A[r][q], __dmul_rn(f, A[c][q]));
+        b[r] = __dsub_rn(b[r], __dmul_rn(f, b[c]));
+      }
+    }
+    if (singular) continue;
+    double x[K];
+#pragma unroll
+    for (int r = K - 1; r >= 0; --r) {
+      double sacc = b[r];
+#pragma unroll
+      for (int q = r + 1; q < K; ++q) sacc = __dsub_rn(sacc, __dmul_rn(A[r][q], x[q]));
+      x[r] = sacc / A[r][r];
+    }
+    // x = tstar * 2^-(S-1); the mantissa of t_j at exponent E is rint(x_j * 2^(S-1-E)).
+    // fits() is monotone in E, so the smallest fitting E is found by stepping
+    // from an estimate.
+    double xm = 0.0;
+#pragma unroll
+    for (int j = 0; j < K; ++j) xm = fmax(xm, fabs(x[j]));
+    int E = (xm > 0.0) ? ((int)((__double_as_longlong(xm) >> 52) & 2047) - 1023) + (S - 1) - 2 : -8;
+    E = E < -8 ? -8 : (E > 7 ? 7 : E);
+    while (E > -8 && fits<K>(x, pow2d(S - 1 - (E - 1)))) --E;
+    while (E < 7 && !fits<K>(x, pow2d(S - 1 - E))) ++E;
+    int t[K];
+    const double sc = pow2d(S - 1 - E);
+#pragma unroll
+    for (int j = 0; j < K; ++j) {
+      double m = rint(__dmul_rn(x[j], sc));
+      m = m < -8.0 ? -8.0 : (m > 7.0 ? 7.0 : m);
+      t[j] = (int)m;
+    }
+    // Quantized squared error, summed in i order.
+    const double vs = pow2d(1 - S + E);
+    double err = 0.0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      int Ri = 0;
+#pragma unroll
+      for (int j = 0; j < K; ++j) Ri += u[i][j] * t[j];
+      const double d = __dsub_rn(w[i], __dmul_rn((double)Ri, vs));
+      err = __dadd_rn(err, __dmul_rn(d, d));
+    }
+    if (err < best) {
+      best = err;
+      bseed = s;
+      bE = E;
+#pragma unroll
+      for (int j = 0; j < K; ++j) bt[j] = t[j];
+    }
+  }
+}
+
+// Warp reduction: smallest error, ties to the smaller seed (the first minimum
+// of an ascending scan).  Lane 0 ends with the winner.
+__device__ __forceinline__ void warp_best(double &best, uint32_t &bseed, int &bE, int (&bt)[6]) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    const double ob = __shfl_down_sync(0xffffffffu, best, off);
+    const uint32_t os = __shfl_down_sync(0xffffffffu, bseed, off);
+    const int oE = __shfl_down_sync(0xffffffffu, bE, off);
+    int ot[6];
+#pragma unroll
+    for (int j = 0; j < 6; ++j) ot[j] = __shfl_down_sync(0xffffffffu, bt[j], off);
+    const bool take = (os != 0) && (bseed == 0 || ob < best || (ob == best && os < bseed));
+    if (take) {
+      best = ob;
+      bseed = os;
+      bE = oE;
+#pragma unroll
+      for (int j = 0; j < 6; ++j) bt[j] = ot[j];
+    }
+  }
+}
+
+struct EncodeOut {
+  uint32_t *seed;
+  int8_t *E;
+  int8_t *t;   // 6 per block
+  double *err;
+};
+
+__device__ __forceinline__ void write_out(const EncodeOut &o, int64_t blk, double best, uint32_t bseed,
+                                          int bE, const int (&bt)[6], int K) {
+  o.seed[blk] = bseed;
+  o.E[blk] = (int8_t)bE;
+  for (int j = 0; j < 6; ++j) o.t[blk * 6 + j] = (int8_t)(j < K ? bt[j] : 0);
+  if (o.err) o.err[blk] = best;
+}
+
+template <int K>
+__device__ __forceinline__ void encode_one(int S, const uint64_t *tab, const double (&w)[8], int lane,
+                                           const EncodeOut &o, int64_t blk) {
+  double best;
+  uint32_t bseed;
+  int bE, bt[6];
+  search_block<K>(S, tab, w, lane, best, bseed, bE, bt);
+  warp_best(best, bseed, bE, bt);
+  if (lane == 0) write_out(o, blk, best, bseed, bE, bt, K);
+}
+
+__device__ __forceinline__ void encode_dispatch(int S, int K, const uint64_t *tab, const double (&w)[8],
+                                                int lane, const EncodeOut &o, int64_t blk) {
+  switch (K) {
+    case 2: encode_one<2>(S, tab, w, lane, o, blk); break;
+    case 3: encode_one<3>(S, tab, w, lane, o, blk); break;
+    case 4: encode_one<4>(S, tab, w, lane, o, blk); break;
+    case 5: encode_one<5>(S, tab, w, lane, o, blk); break;
+    default: encode_one<6>(S, tab, w, lane, o, blk); break;
+  }
+}
+
+// A list of blocks at one rung: w is nblocks x 8 (row-major), fp32.
+__global__ void __launch_bounds__(kEncWarps * 32) k_encode_list(int S, int K, uint32_t taps, const float *w,
+                                                              int64_t nblocks, EncodeOut o) {
+  __shared__ uint64_t tab[512];
+  for (int v = threadIdx.x; v < 512; v += blockDim.x) tab[v] = jump_table_entry(S, taps, v);
+  __syncthreads();
+  const int lane = threadIdx.x & 31;
+  for (int64_t blk = (int64_t)blockIdx.x * kEncWarps + (threadIdx.x >> 5); blk < nblocks;
+       blk += (int64_t)gridDim.x * kEncWarps) {
+    double wv[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) wv[i] = (double)__ldg(w + blk * 8 + i);
+    encode_dispatch(S, K, tab, wv, lane, o, blk);
+  }
+}
+
+// Every block of a prepared layer at the rung its plan assigns: W is R x C
+// fp32 in the original column order; block (r, c) holds W[r, perm[8c + i]].
+__global__ void __launch_bounds__(kEncWarps * 32) k_encode_layer(const __grid_constant__ LayerArgs p,
+                                                               const float *W, EncodeOut o) {
+  extern __shared__ uint64_t tabs[];  // nslots x 512
+  for (int v = threadIdx.x; v < p.nslots * 512; v += blockDim.x) tabs[v] = __ldg(p.tables + v);
+  __syncthreads();
+  const int lane = threadIdx.x & 31;
+  const int64_t total = p.R * (int64_t)p.nb;
+  for (int64_t blk = (int64_t)blockIdx.x * kEncWarps + (threadIdx.x >> 5); blk < total;
+       blk += (int64_t)gridDim.x * kEncWarps) {
+    const int64_t r = blk / p.nb;
+    const int c = (int)(blk - r * p.nb);
+    int32_t bk[kMaxJ];
+    for (int j = 0; j < p.J - 1; ++j) bk[j] = __ldg(p.brk + r * (p.J - 1) + j);
+    const int g = rung_of(bk, p.J, c);
+    double wv[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) wv[i] = (double)__ldg(W + r * p.C + __ldg(p.perm + 8 * c + i));
+    encode_dispatch(rung_S(p.code[g]), rung_K(p.code[g]), tabs + (size_t)p.slot[g] * 512, wv, lane, o, blk);
+  }
+}
+
+// Pack the fields of every block at its bit offset (one thread per block).
+__global__ void k_pack(const __grid_constant__ LayerArgs p, const uint32_t *seed, const int8_t *E,
+                       const int8_t *t, uint32_t *out) {
+  const int64_t total = p.R * (int64_t)p.nb;
+  for (int64_t b = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; b < total;
+       b += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t r = b / p.nb;
+    const int c = (int)(b - r * p.nb);
+    int32_t bk[kMaxJ];
+    for (int j = 0; j < p.J - 1; ++j) bk[j] = p.brk[r * (p.J - 1) + j];
+    const int g = rung_of(bk, p.J, c);
+    const int S = rung_S(p.code[g]), K = rung_K(p.code[g]);
+    const uint64_t off = p.row_off[r] + bits_before(bk, p.J, p.L, p.nb, c);
+    uint64_t v = (uint64_t)(seed[b] & ((1u << S) - 1u)) | ((uint64_t)(E[b] & 15) << S);
+    for (int j = 0; j < K; ++j) v |= (uint64_t)(t[b * 6 + j] & 15) << (S + 4 + 4 * j);
+    const uint64_t wi = off >> 5;
+    const int sh = (int)(off & 31);
+    atomicOr(out + wi, (uint32_t)(v << sh));
+    const uint64_t rest = (sh == 0) ? (v >> 32) : (v >> (32 - sh));
+    if (rest) atomicOr(out + wi + 1, (uint32_t)rest);
+    const uint64_t rest2 = (sh == 0) ? 0 : (v >> (64 - sh));
+    if (sh && rest2) atomicOr(out + wi + 2, (uint32_t)rest2);
+  }
+}
+
+static int grid_for(int64_t nblocks) {
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t want = (nblocks + kEncWarps - 1) / kEncWarps;
+  const int64_t cap = (int64_t)(sms > 0 ? sms : 1) * 16;
+  return (int)(want < cap ? (want > 0 ? want : 1) : cap);
+}
+
+}  // namespace seedq
+
+using namespace seedq;
+
+extern "C" {
+
+seedq_status seedq_encode_blocks(int32_t S, int32_t k, const float *w, int64_t nblocks, uint32_t *seed,
+                                 int8_t *E, int8_t *t, double *err, void *cuda_stream) {
+  if (S < 8 || S > 16 || (S & 1) || k < 2 || k > 6) return SEEDQ_ERR_UNSUPPORTED;
+  if (nblocks < 0 || (nblocks > 0 && (!w || !seed || !E || !t))) return SEEDQ_ERR_INVALID_ARG;
+  if (nblocks == 0) return SEEDQ_OK;
+  EncodeOut o{seed, E, t, err};
+  k_encode_list<<<grid_for(nblocks), kEncWarps * 32, 0, (cudaStream_t)cuda_stream>>>(
+      S, k, seedq_lfsr_taps(S), w, nblocks, o);
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? SEEDQ_OK : cuda_fail(e);
+}
+
+seedq_status seedq_encode_layer(const seedq_layer *L, const float *W, uint32_t *seed, int8_t *E, int8_t *t,
+                                double *err, void *cuda_stream) {
+  if (!L || !W || !seed || !E || !t) return SEEDQ_ERR_INVALID_ARG;
+  const int64_t total = L->args.R * (int64_t)L->args.nb;
+  EncodeOut o{seed, E, t, err};
+  const size_t smem = sizeof(uint64_t) * 512 * (size_t)L->args.nslots;
+  k_encode_layer<<<grid_for(total), kEncWarps * 32, smem, (cudaStream_t)cuda_stream>>>(L->args, W, o);
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? SEEDQ_OK : cuda_fail(e);
+}
+
+seedq_status seedq_pack_stream(const seedq_layer *L, const uint32_t *seed, const int8_t *E, const int8_t *t,
+                               void *stream, uint64_t stream_bytes, void *cuda_stream) {
+  if (!L || !seed || !E || !t || !stream || ((uintptr_t)stream & 15u)) return SEEDQ_ERR_INVALID_ARG;
+  if (stream_bytes < stream_bytes_required(L->total_bits)) return SEEDQ_ERR_STREAM;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  cudaError_t e = cudaMemsetAsync(stream, 0, stream_bytes, st);
+  if (e == cudaSuccess) {
+    const int64_t total = L->args.R * (int64_t)L->args.nb;
+    const int64_t want = (total + 255) / 256;
+    k_pack<<<(int)(want < 4096 ? (want > 0 ? want : 1) : 4096), 256, 0, st>>>(L->args, seed, E, t,
+                                                                             (uint32_t *)stream);
+    e = cudaGetLastError();
+  }
+  return e == cudaSuccess ? SEEDQ_OK : cuda_fail(e);
+}
+
+}  // extern "C"

@@ -243,15 +243,7 @@ __global__ void k_tables(const int32_t *__restrict__ slot_S, uint64_t *__restric
   const int S = slot_S[slot];
   const uint32_t taps = taps_arr[S - 8];
   const int v = threadIdx.x;  // 0..511
-  const uint32_t seed = (v < 256) ? (uint32_t)v : ((uint32_t)(v - 256) << 8);
-  uint64_t q = (uint64_t)(seed & ((1u << S) - 1u));
-  if (v >= 256 && S <= 8) q = 0;
-  for (int t = S; t < 64; ++t) {
-    const uint64_t win = (q >> (t - S)) & (uint64_t)taps;
-    const uint64_t bit = (uint64_t)(__popcll(win) & 1);
-    q |= bit << t;
-  }
-  tables[(size_t)slot * 512 + v] = q;
+  tables[(size_t)slot * 512 + v] = jump_table_entry(S, taps, v);
 }
 
 // Synthetic payload of the workload recipe, one thread per block.

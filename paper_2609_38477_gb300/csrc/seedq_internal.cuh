@@ -135,6 +135,23 @@ __device__ __forceinline__ int rung_of(const int32_t *b, int J, int c) {
   return j;
 }
 
+// Entry v of the GF(2) jump table of width S (0 <= v < 512): the first 64
+// sequence bits o_0..o_63 from seed v (v < 256) or from seed (v - 256) << 8
+// reduced to S bits (zero for S = 8), by the window recurrence
+// o_{t+S} = XOR over set bits i of taps of o_{t+i}.  By linearity the prefix
+// of any seed s is tab[s & 255] ^ tab[256 + (s >> 8)].
+__device__ __forceinline__ uint64_t jump_table_entry(int S, uint32_t taps, int v) {
+  const uint32_t seed = (v < 256) ? (uint32_t)v : ((uint32_t)(v - 256) << 8);
+  uint64_t q = (uint64_t)(seed & ((1u << S) - 1u));
+  if (v >= 256 && S <= 8) q = 0;
+  for (int t = S; t < 64; ++t) {
+    const uint64_t win = (q >> (t - S)) & (uint64_t)taps;
+    const uint64_t bit = (uint64_t)(__popcll(win) & 1);
+    q |= bit << t;
+  }
+  return q;
+}
+
 // 64 stream bits starting at bit `off`: lo = bits [off, off+32), hi = [off+32, off+64).
 template <int NWORDS>
 __device__ __forceinline__ void load_bits(const uint32_t *__restrict__ w, uint64_t off,

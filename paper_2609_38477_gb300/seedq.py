@@ -71,6 +71,12 @@ SIGNATURES = {
     "seedq_row_plan_static": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int64, C.c_int32,
                                         C.POINTER(Schedule), C.c_int64, C.c_void_p, C.c_void_p,
                                         C.c_void_p, C.c_void_p]),
+    "seedq_encode_blocks": (C.c_int, [C.c_int32, C.c_int32, C.c_void_p, C.c_int64, C.c_void_p,
+                                      C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
+    "seedq_encode_layer": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                                     C.c_void_p, C.c_void_p]),
+    "seedq_pack_stream": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                                    C.c_uint64, C.c_void_p]),
     "seedq_status_string": (C.c_char_p, [C.c_int]),
     "seedq_last_cuda_error_string": (C.c_char_p, []),
 }
@@ -192,6 +198,14 @@ class Layer:
         _check(lib().seedq_gemm_small_batch(self.h, _ptr(X), n, _ptr(Y), _stream(stream)),
                "seedq_gemm_small_batch")
 
+    def encode(self, W, seed, E, t, err=None, stream=None):
+        _check(lib().seedq_encode_layer(self.h, _ptr(W), _ptr(seed), _ptr(E), _ptr(t), _ptr(err),
+                                        _stream(stream)), "seedq_encode_layer")
+
+    def pack_stream(self, seed, E, t, buf, nbytes: int, stream=None):
+        _check(lib().seedq_pack_stream(self.h, _ptr(seed), _ptr(E), _ptr(t), _ptr(buf), nbytes,
+                                       _stream(stream)), "seedq_pack_stream")
+
     # -- introspection (synchronous) --------------------------------------
     def rung_map(self, row0: int = 0, nrows: int | None = None) -> np.ndarray:
         nrows = self.rows - row0 if nrows is None else nrows
@@ -236,3 +250,9 @@ def gemm_multi(layers, X, n: int, Y, stream=None):
     xh = (C.c_void_p * cnt)(*[_ptr(x) for x in X])
     yh = (C.c_void_p * cnt)(*[_ptr(y) for y in Y])
     _check(lib().seedq_gemm_multi(lh, cnt, xh, n, yh, _stream(stream)), "seedq_gemm_multi")
+
+
+def encode_blocks(S: int, k: int, w, nblocks: int, seed, E, t, err=None, stream=None):
+    """seedq_encode_blocks: exhaustive seed search of nblocks blocks at rung (S, k)."""
+    _check(lib().seedq_encode_blocks(S, k, _ptr(w), nblocks, _ptr(seed), _ptr(E), _ptr(t), _ptr(err),
+                                     _stream(stream)), "seedq_encode_blocks")
