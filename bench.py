@@ -31,13 +31,24 @@ FLUSH_BYTES = 512 << 20  # > 129 MB L2: written between timed steps
 def parse():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=2000)
-    p.add_argument("--warmup", type=int, default=10)
+    p.add_argument("--steps", type=int, default=None,
+                   help="timed steps (default 2000 for the fused GEMV, 5 for the encoder)")
+    p.add_argument("--warmup", type=int, default=None)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default="c1")
     p.add_argument("--batch", type=int, default=1)
     p.add_argument("--no-cpu-baseline", action="store_true")
-    return p.parse_args()
+    p.add_argument("--path", choices=["gemv", "encode"], default="gemv",
+                   help="gemv: the fused decode + GEMV step (default); encode: the exhaustive "
+                        "seed-search encoder")
+    p.add_argument("--rung", default="16,3", help="encoder rung S,k")
+    p.add_argument("--blocks", type=int, default=4864, help="encoder blocks per step")
+    a = p.parse_args()
+    if a.steps is None:
+        a.steps = 2000 if a.path == "gemv" else 5
+    if a.warmup is None:
+        a.warmup = 10 if a.path == "gemv" else 3
+    return a
 
 
 def load_schedule(name):
@@ -436,9 +447,192 @@ def our_arm(args):
         gt.layer.release()
 
 
+# ------------------------------------------------------------ encoder path
+
+ENC_METRIC = "encoder blocks/s (exhaustive seed search, Sec. 3.1)"
+
+
+def encode_inputs(S, k, nblocks):
+    """Synthetic weight blocks, w ~ N(0, 0.02^2), seeded; the encoder's work does
+    not depend on the values beyond the rare singular seed."""
+    import numpy as np
+    from paper_2609_38477_gb300 import workloads as W
+
+    w = 0.02 * W.normal(W.derive_key(5, 17, S, k), nblocks * 8)
+    return np.ascontiguousarray(w.astype(np.float32).reshape(nblocks, 8))
+
+
+def encode_flops_per_seed(k):
+    """fp64 operations of one seed's fit as the search performs them: the
+    right-hand side (8 products and 8 sums per coefficient), the elimination
+    and back substitution (one division, product and difference per entry
+    touched), two exponent probes (one product per mantissa), the mantissas,
+    and the error (a product by the exponent, a difference, a square and a
+    sum per weight)."""
+    rhs = 16 * k
+    elim = sum((k - 1 - c) * (1 + 2 * (k - 1 - c) + 2) for c in range(k))
+    back = sum(1 + 2 * (k - 1 - r) for r in range(k))
+    return rhs + elim + back + 3 * k + 4 * 8
+
+
+def encode_oracle_sample(S, k, w, target_s, nthreads):
+    sys.path.insert(0, os.path.join(ROOT, "oracle"))
+    import concurrent.futures as cf
+
+    import oracle as O
+
+    taps = O.find_taps(S)
+    t0 = time.perf_counter()
+    O.encode_block(S, k, taps, w[0].astype("float64"))
+    per = max(time.perf_counter() - t0, 1e-6)
+    n = int(max(nthreads, min(len(w), target_s * nthreads / per)))
+    n = min(n, len(w))
+
+    def run():
+        with cf.ThreadPoolExecutor(nthreads) as ex:
+            list(ex.map(lambda b: O.encode_block(S, k, taps, w[b].astype("float64")), range(n)))
+        return n
+
+    return run, n
+
+
+def encode_reference(args):
+    if int(os.environ.get("RANK", "0")) != 0:
+        return
+    S, k = (int(v) for v in args.rung.split(","))
+    w = encode_inputs(S, k, args.blocks)
+    cores = cpu_cores()
+    run, n = encode_oracle_sample(S, k, w, max(0.2, min(6.0, 60.0 / max(args.steps + args.warmup, 1))),
+                                  cores)
+    for _ in range(args.warmup):
+        run()
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        run()
+        times.append(time.perf_counter() - t0)
+    value = n / statistics.mean(times)
+    desc = f"oracle seed search of {n} of the {args.blocks} blocks on {cores} host threads"
+    print(json.dumps({
+        "impl": "reference", "metric": ENC_METRIC, "value": value, "unit": "blocks/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": statistics.mean(times) * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": f"exhaustive seed search at rung ({S},{k}), {args.blocks} blocks"},
+        "cpu_baseline": {"value": value, "unit": "blocks/s", "cores": cores, "kind": "oracle",
+                         "sample": desc},
+        "e2e": {"value": value, "unit": "blocks/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+def encode_arm(args):
+    import numpy as np
+    import torch
+
+    rank, world, local = dist_init()
+    torch.cuda.set_device(local)
+    import __graft_entry__ as GE
+
+    GE.build()
+    from paper_2609_38477_gb300 import seedq as Q
+
+    S, k = (int(v) for v in args.rung.split(","))
+    nb = args.blocks
+    w = encode_inputs(S, k, nb)
+    wd = torch.from_numpy(w).cuda()
+    seed = torch.empty(nb, dtype=torch.int32, device="cuda")
+    E = torch.empty(nb, dtype=torch.int8, device="cuda")
+    t = torch.empty(nb * 6, dtype=torch.int8, device="cuda")
+    err = torch.empty(nb, dtype=torch.float64, device="cuda")
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.current_stream()
+    h = stream.cuda_stream
+
+    def step():
+        Q.encode_blocks(S, k, wd, nb, seed, E, t, err, h)
+
+    for _ in range(max(args.warmup, 3)):
+        flush.zero_()
+        step()
+    torch.cuda.synchronize()
+    clocks = Clocks(gpu_index(local))
+    dist_barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    for a, b in ev:
+        flush.zero_()
+        a.record(stream)
+        step()
+        b.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    dist_barrier()
+    step_ms = dist_max(statistics.mean(a.elapsed_time(b) for a, b in ev))
+
+    # End to end through the C ABI: weights copied in, fields copied out.
+    wh = torch.from_numpy(w).pin_memory()
+    outs = [torch.empty(x.shape, dtype=x.dtype).pin_memory() for x in (seed, E, t, err)]
+    e2e = []
+    for _ in range(args.steps):
+        flush.zero_()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        wd.copy_(wh, non_blocking=True)
+        step()
+        for o, x in zip(outs, (seed, E, t, err)):
+            o.copy_(x, non_blocking=True)
+        b.record(stream)
+        b.synchronize()
+        e2e.append(a.elapsed_time(b))
+    e2e_ms = dist_max(statistics.mean(e2e))
+
+    nseeds = (1 << S) - 1
+    flops = encode_flops_per_seed(k) * nseeds * nb
+    achieved = flops / (step_ms * 1e-3) / 1e12
+    peak = 1.25  # TFLOP/s fp64, nominal (no measured fp64 peak)
+    line = {
+        "metric": ENC_METRIC, "value": world * nb / (step_ms * 1e-3), "unit": "blocks/s",
+        "n_gpus": world, "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": step_ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": f"exhaustive seed search at rung ({S},{k}): {nb} blocks of "
+                               f"w ~ N(0, 0.02^2), {nseeds} seeds each",
+                   "l2": f"flushed between timed steps ({FLUSH_BYTES >> 20} MiB write)"},
+        "seeds_per_s": world * nb * nseeds / (step_ms * 1e-3),
+        "clocks": clk,
+        "e2e": {"value": world * nb / (e2e_ms * 1e-3), "unit": "blocks/s",
+                "h2d_bytes_per_step": w.nbytes,
+                "d2h_bytes_per_step": sum(x.numel() * x.element_size() for x in (seed, E, t, err))},
+        "gpu_launches": args.steps,
+        "roofline": {"bound": "alu", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak, "traffic": None, "kernel": "k_encode_list",
+                     "peak_basis": "fp64 1.25 TFLOP/s nominal (the profiling recipe's table; "
+                                   "MEASURED_PEAKS.json has no fp64 figure)",
+                     "flops_per_seed": encode_flops_per_seed(k)},
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        run, n = encode_oracle_sample(S, k, w, 10.0, cpu_cores())
+        t0 = time.perf_counter()
+        run()
+        dt = time.perf_counter() - t0
+        line["cpu_baseline"] = {"value": n / dt, "unit": "blocks/s", "cores": cpu_cores(),
+                                "kind": "oracle",
+                                "sample": f"oracle seed search of {n} of the {nb} blocks, "
+                                          f"one block per host thread at a time"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
-    if args.impl == "reference":
+    if args.path == "encode":
+        if args.impl == "reference":
+            encode_reference(args)
+        else:
+            encode_arm(args)
+    elif args.impl == "reference":
         reference_arm(args)
     else:
         our_arm(args)

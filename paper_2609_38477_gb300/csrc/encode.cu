@@ -22,6 +22,14 @@
 //
 // Work split: one warp per block, lanes striding over the seeds, then a warp
 // reduction on (error, seed).
+//
+// The fp64 pipe is the bottleneck (a small fraction of the integer pipes'
+// rate), so every step whose result is exact is done with integer
+// instructions on the IEEE bit patterns instead: integers and exact products
+// are converted to doubles by building their bits, products by powers of two
+// add to the exponent field, and comparisons of magnitudes compare bit
+// patterns.  Only the rounded steps (sums, products and quotients of the
+// solve, the error) run on the fp64 pipe.
 #include "seedq_internal.cuh"
 
 namespace seedq {
@@ -31,27 +39,79 @@ constexpr int kEncWarps = 8;
 // Power of two 2^e as a double (|e| well inside the normal range).
 __device__ __forceinline__ double pow2d(int e) { return __longlong_as_double((long long)(1023 + e) << 52); }
 
-// All k rounded mantissas of tstar * 2^-E lie in [-8, 7].
+// The double equal to the integer +-mag * 2^e (mag < 2^63), built from bits.
+__device__ __forceinline__ double exact_d(bool neg, unsigned long long mag, int e) {
+  if (mag == 0) return 0.0;
+  const int msb = 63 - __clzll((long long)mag);
+  const unsigned long long mant = (msb <= 52 ? (mag << (52 - msb)) : (mag >> (msb - 52))) & ((1ull << 52) - 1);
+  return __longlong_as_double((long long)(((unsigned long long)neg << 63) |
+                                          ((unsigned long long)(1023 + msb + e) << 52) | mant));
+}
+__device__ __forceinline__ double i2d(long long v) {
+  return exact_d(v < 0, (unsigned long long)(v < 0 ? -v : v), 0);
+}
+// |bits| of a double, as an integer whose order is the order of magnitudes.
+__device__ __forceinline__ unsigned long long mag_bits(double d) {
+  return (unsigned long long)__double_as_longlong(d) & 0x7fffffffffffffffull;
+}
+// d * 2^e for d normal or zero (exponent field shift).
+__device__ __forceinline__ double scale2(double d, int e) {
+  const long long b = __double_as_longlong(d);
+  return (b & 0x7fffffffffffffffll) == 0 ? d : __longlong_as_double(b + ((long long)e << 52));
+}
+
+// All k round-half-even values of x_j * 2^e lie in [-8, 7], i.e. every
+// x_j * 2^e lies in [-8.5, 7.5) (compared as bit patterns: exact).
 template <int K>
-__device__ __forceinline__ bool fits(const double (&ts)[K], double scale) {
+__device__ __forceinline__ bool fits(const double (&x)[K], int e) {
+  const unsigned long long lim_neg = (unsigned long long)__double_as_longlong(8.5);
+  const unsigned long long lim_pos = (unsigned long long)__double_as_longlong(7.5);
   bool ok = true;
 #pragma unroll
   for (int j = 0; j < K; ++j) {
-    const double m = rint(__dmul_rn(ts[j], scale));
-    ok = ok && (m >= -8.0) && (m <= 7.0);
+    const double v = scale2(x[j], e);
+    const unsigned long long b = (unsigned long long)__double_as_longlong(v);
+    ok = ok && ((b >> 63) ? ((b & 0x7fffffffffffffffull) <= lim_neg) : (b < lim_pos));
   }
   return ok;
 }
 
 // Search all seeds of one block (w: 8 weights) for the lane's share of seeds.
 // Returns the lane's best (error, seed, E, t) in the order of the scan.
-template <int K>
-__device__ __forceinline__ void search_block(int S, const uint64_t *tab, const double (&w)[8], int lane,
+template <int K, bool kExactRhs>
+__device__ __forceinline__ void search_block(int S, const uint64_t *tab, const float (&wf)[8], int lane,
                                              double &best, uint32_t &bseed, int &bE, int (&bt)[6]) {
+  // Each weight as +-mw * 2^ew with an integer mantissa (exact for floats).
+  double w[8];
+  bool wneg[8];
+  unsigned int wm[8];
+  int we[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    w[i] = (double)wf[i];
+    const unsigned int fb = __float_as_uint(wf[i]);
+    const int ef = (int)((fb >> 23) & 255u);
+    wneg[i] = (fb >> 31) != 0;
+    wm[i] = (fb & 0x7fffffu) | (ef ? 0x800000u : 0u);
+    we[i] = (ef ? ef : 1) - 150;
+  }
+  // Right-hand side without rounding: when the weights' exponents lie within
+  // 11 of each other, every product |u| * mw (< 2^39) aligned to the smallest
+  // exponent stays below 2^50, so every partial sum of the eight is an integer
+  // below 2^53: each fp64 addition of the sequence is then exact, and the sum
+  // equals the integer sum (the caller picks this variant per block).
+  int emin = 1 << 20;
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+    if (wm[i]) emin = min(emin, we[i]);
+  if (emin == (1 << 20)) emin = 0;  // all weights zero
+  int wsh[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) wsh[i] = wm[i] ? we[i] - emin : 0;
   const uint32_t mask = (1u << S) - 1u;
   const int h = 1 << (S - 1);
   // Pivot threshold of the unscaled matrix: 1e-12 * 2^(2S-2), exact.
-  const double thr = __dmul_rn(1e-12, pow2d(2 * S - 2));
+  const unsigned long long thr = mag_bits(__dmul_rn(1e-12, pow2d(2 * S - 2)));
   best = __longlong_as_double(0x7ff0000000000000ll);  // +inf
   bseed = 0;
   bE = 0;
@@ -69,16 +129,32 @@ __device__ __forceinline__ void search_block(int S, const uint64_t *tab, const d
     double A[K][K], b[K];
 #pragma unroll
     for (int p = 0; p < K; ++p) {
-      double r = 0.0;
+      if constexpr (kExactRhs) {
+        long long acc = 0;
 #pragma unroll
-      for (int i = 0; i < 8; ++i) r = __dadd_rn(r, __dmul_rn((double)u[i][p], w[i]));
-      b[p] = r;
+        for (int i = 0; i < 8; ++i) {
+          const long long pr = ((long long)u[i][p] * (long long)wm[i]) << wsh[i];
+          acc += wneg[i] ? -pr : pr;
+        }
+        b[p] = exact_d(acc < 0, (unsigned long long)(acc < 0 ? -acc : acc), emin);
+      } else {
+        double r = 0.0;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          // u * w is exact: built from the integer product of the mantissas.
+          const int ui = u[i][p];
+          const double prod = exact_d(wneg[i] != (ui < 0),
+                                      (unsigned long long)(ui < 0 ? -ui : ui) * wm[i], we[i]);
+          r = __dadd_rn(r, prod);
+        }
+        b[p] = r;
+      }
 #pragma unroll
       for (int q = p; q < K; ++q) {
         long long acc = 0;
 #pragma unroll
         for (int i = 0; i < 8; ++i) acc += (long long)(u[i][p] * u[i][q]);
-        A[p][q] = (double)acc;
+        A[p][q] = i2d(acc);
         A[q][p] = A[p][q];
       }
     }
@@ -87,10 +163,10 @@ __device__ __forceinline__ void search_block(int S, const uint64_t *tab, const d
 #pragma unroll
     for (int c = 0; c < K; ++c) {
       int pr = c;
-      double pv = fabs(A[c][c]);
+      unsigned long long pv = mag_bits(A[c][c]);
 #pragma unroll
       for (int r = c + 1; r < K; ++r) {
-        const double v = fabs(A[r][c]);
+        const unsigned long long v = mag_bits(A[r][c]);
         if (v > pv) {
           pv = v;
           pr = r;
@@ -131,30 +207,28 @@ __device__ __forceinline__ void search_block(int S, const uint64_t *tab, const d
     // x = tstar * 2^-(S-1); the mantissa of t_j at exponent E is rint(x_j * 2^(S-1-E)).
     // fits() is monotone in E, so the smallest fitting E is found by stepping
     // from an estimate.
-    double xm = 0.0;
+    unsigned long long xm = 0;
 #pragma unroll
-    for (int j = 0; j < K; ++j) xm = fmax(xm, fabs(x[j]));
-    int E = (xm > 0.0) ? ((int)((__double_as_longlong(xm) >> 52) & 2047) - 1023) + (S - 1) - 2 : -8;
+    for (int j = 0; j < K; ++j) xm = max(xm, mag_bits(x[j]));
+    int E = xm ? ((int)(xm >> 52) - 1023) + (S - 1) - 2 : -8;
     E = E < -8 ? -8 : (E > 7 ? 7 : E);
-    while (E > -8 && fits<K>(x, pow2d(S - 1 - (E - 1)))) --E;
-    while (E < 7 && !fits<K>(x, pow2d(S - 1 - E))) ++E;
+    while (E > -8 && fits<K>(x, S - 1 - (E - 1))) --E;
+    while (E < 7 && !fits<K>(x, S - 1 - E)) ++E;
     int t[K];
-    const double sc = pow2d(S - 1 - E);
 #pragma unroll
     for (int j = 0; j < K; ++j) {
-      double m = rint(__dmul_rn(x[j], sc));
+      double m = rint(scale2(x[j], S - 1 - E));
       m = m < -8.0 ? -8.0 : (m > 7.0 ? 7.0 : m);
       t[j] = (int)m;
     }
     // Quantized squared error, summed in i order.
-    const double vs = pow2d(1 - S + E);
     double err = 0.0;
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       int Ri = 0;
 #pragma unroll
       for (int j = 0; j < K; ++j) Ri += u[i][j] * t[j];
-      const double d = __dsub_rn(w[i], __dmul_rn((double)Ri, vs));
+      const double d = __dsub_rn(w[i], exact_d(Ri < 0, (unsigned long long)(Ri < 0 ? -Ri : Ri), 1 - S + E));
       err = __dadd_rn(err, __dmul_rn(d, d));
     }
     if (err < best) {
@@ -205,17 +279,30 @@ __device__ __forceinline__ void write_out(const EncodeOut &o, int64_t blk, doubl
 }
 
 template <int K>
-__device__ __forceinline__ void encode_one(int S, const uint64_t *tab, const double (&w)[8], int lane,
+__device__ __forceinline__ void encode_one(int S, const uint64_t *tab, const float (&w)[8], int lane,
                                            const EncodeOut &o, int64_t blk) {
   double best;
   uint32_t bseed;
   int bE, bt[6];
-  search_block<K>(S, tab, w, lane, best, bseed, bE, bt);
+  // Exponent spread of the block's weights (zeros do not constrain it).
+  int emin = 1 << 20, emax = -(1 << 20);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const unsigned int fb = __float_as_uint(w[i]);
+    if (fb & 0x7fffffffu) {
+      const int ef = (int)((fb >> 23) & 255u);
+      const int e = (ef ? ef : 1) - 150;
+      emin = min(emin, e);
+      emax = max(emax, e);
+    }
+  }
+  if (emax - emin <= 11) search_block<K, true>(S, tab, w, lane, best, bseed, bE, bt);
+  else search_block<K, false>(S, tab, w, lane, best, bseed, bE, bt);
   warp_best(best, bseed, bE, bt);
   if (lane == 0) write_out(o, blk, best, bseed, bE, bt, K);
 }
 
-__device__ __forceinline__ void encode_dispatch(int S, int K, const uint64_t *tab, const double (&w)[8],
+__device__ __forceinline__ void encode_dispatch(int S, int K, const uint64_t *tab, const float (&w)[8],
                                                 int lane, const EncodeOut &o, int64_t blk) {
   switch (K) {
     case 2: encode_one<2>(S, tab, w, lane, o, blk); break;
@@ -235,9 +322,9 @@ __global__ void __launch_bounds__(kEncWarps * 32) k_encode_list(int S, int K, ui
   const int lane = threadIdx.x & 31;
   for (int64_t blk = (int64_t)blockIdx.x * kEncWarps + (threadIdx.x >> 5); blk < nblocks;
        blk += (int64_t)gridDim.x * kEncWarps) {
-    double wv[8];
+    float wv[8];
 #pragma unroll
-    for (int i = 0; i < 8; ++i) wv[i] = (double)__ldg(w + blk * 8 + i);
+    for (int i = 0; i < 8; ++i) wv[i] = __ldg(w + blk * 8 + i);
     encode_dispatch(S, K, tab, wv, lane, o, blk);
   }
 }
@@ -258,9 +345,9 @@ __global__ void __launch_bounds__(kEncWarps * 32) k_encode_layer(const __grid_co
     int32_t bk[kMaxJ];
     for (int j = 0; j < p.J - 1; ++j) bk[j] = __ldg(p.brk + r * (p.J - 1) + j);
     const int g = rung_of(bk, p.J, c);
-    double wv[8];
+    float wv[8];
 #pragma unroll
-    for (int i = 0; i < 8; ++i) wv[i] = (double)__ldg(W + r * p.C + __ldg(p.perm + 8 * c + i));
+    for (int i = 0; i < 8; ++i) wv[i] = __ldg(W + r * p.C + __ldg(p.perm + 8 * c + i));
     encode_dispatch(rung_S(p.code[g]), rung_K(p.code[g]), tabs + (size_t)p.slot[g] * 512, wv, lane, o, blk);
   }
 }

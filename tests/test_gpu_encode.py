@@ -40,6 +40,11 @@ def _blocks(rng, n, S, k):
         E = int(rng.integers(-8, -2))
         t = rng.integers(-8, 8, k).tolist()
         w[i] = O.reconstruct_block(S, k, taps, seed, E, t)
+    if n > 6:
+        # Wide exponent spread (the rounded right-hand-side path) and a block
+        # with zero entries and a subnormal (the exact path).
+        w[4] = np.array([3e-7, -0.05, 0.02, 1e-5, -0.03, 0.011, -2e-6, 0.04], np.float32)
+        w[5] = np.array([0.0, -0.01, 0.0, 0.013, 1e-40, -0.02, 0.0, 0.008], np.float32)
     return w
 
 
