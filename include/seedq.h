@@ -47,7 +47,9 @@ typedef enum {
   SEEDQ_ERR_SCHEDULE = 3,     /* thresholds not increasing, tie count > tied blocks */
   SEEDQ_ERR_CUDA = 4,         /* a CUDA runtime call failed */
   SEEDQ_ERR_NOMEM = 5,        /* device or host allocation failed (prepare only) */
-  SEEDQ_ERR_UNSUPPORTED = 6   /* rung or shape outside what the kernels implement */
+  SEEDQ_ERR_UNSUPPORTED = 6,  /* rung or shape outside what the kernels implement */
+  SEEDQ_ERR_IO = 7,           /* a container file could not be opened, read or written */
+  SEEDQ_ERR_FORMAT = 8        /* a container file is malformed, truncated or corrupted */
 } seedq_status;
 
 /* A rung g = (S, k) of the hull: seed width S and coefficient count k (Sec. 3.1).
@@ -227,6 +229,50 @@ seedq_status seedq_encode_layer(const seedq_layer *layer, const float *W, uint32
 seedq_status seedq_pack_stream(const seedq_layer *layer, const uint32_t *seed, const int8_t *E,
                                const int8_t *t, void *stream, uint64_t stream_bytes,
                                void *cuda_stream);
+
+/* -------------------------------------------------------------- container
+ * A file holding a compressed model: the global decoder table (Sec. 3.6, as
+ * seedq_schedule) and, per tensor, what Alg. 2 reads besides it: shape,
+ * importance factors a and rho (the decoder recomputes the rung map from
+ * them), T_t, the FP16 outlier columns (Sec. 3.5) and the payload stream.
+ * Little-endian, no padding; the header records the LFSR taps of S = 8..16
+ * (a file written with other taps is rejected with SEEDQ_ERR_UNSUPPORTED) and
+ * the file ends in a 64-bit FNV-1a hash of its contents (checked on open).
+ * Host functions; they never touch the GPU.
+ *
+ * Per-tensor view.  All pointers are host memory: on write they are read
+ * only; from seedq_container_get they point into the container and stay valid
+ * until seedq_container_close.  outlier_vals is rows x n_outliers binary16
+ * (host here, unlike seedq_layer_desc, which wants them on the device);
+ * stream holds ceil(stream_bits / 8) bytes. */
+typedef struct {
+  const char *name;
+  int64_t rows;
+  int64_t cols;
+  const float *a;
+  const float *rho;           /* NULL: all ones */
+  int64_t tie_count;
+  int32_t n_outliers;
+  const int32_t *outlier_cols;
+  const uint16_t *outlier_vals;
+  const uint8_t *stream;
+  uint64_t stream_bits;
+} seedq_container_tensor;
+
+typedef struct seedq_container seedq_container;
+
+/* Write the schedule and ntensors tensors to path (replacing the file). */
+seedq_status seedq_container_write(const char *path, const seedq_schedule *sched,
+                                   int32_t ntensors, const seedq_container_tensor *tensors);
+/* Read and validate a container; *out receives it (release with _close).
+ * Errors: IO, FORMAT (bad magic, version, sizes, hash), UNSUPPORTED (taps). */
+seedq_status seedq_container_open(const char *path, seedq_container **out);
+/* The stored schedule; its arrays point into the container. */
+seedq_status seedq_container_schedule(const seedq_container *c, seedq_schedule *sched);
+seedq_status seedq_container_count(const seedq_container *c, int32_t *ntensors);
+seedq_status seedq_container_get(const seedq_container *c, int32_t index,
+                                 seedq_container_tensor *tensor);
+seedq_status seedq_container_close(seedq_container *c);
 
 /* Fill a stream buffer with the synthetic payload of the workload recipe:
  * block b of the tensor (row-major) draws h = splitmix64 output number b from

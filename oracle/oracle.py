@@ -368,3 +368,108 @@ def hull_rungs(damage: dict, rbar: float, band=(1.0, 1.5)):
     rates = [block_bits(S, k) / 8.0 for S, k in rungs]
     slopes = [(es[j] - es[j + 1]) / (rates[j + 1] - rates[j]) for j in range(len(rungs) - 1)]
     return rungs, es, slopes
+
+
+# ------------------------------------------------------------ container file
+# The oracle's own reader and writer of the container layout (the model file
+# holding the Sec. 3.6 table and, per tensor, the inputs of Alg. 2 and the
+# stream): little-endian fields in this order, then a 64-bit FNV-1a hash of
+# all preceding bytes.  Written independently of the library's C++ version.
+
+import struct as _st
+
+_MAGIC = b"SEEDQ\x00v1"
+
+
+def _fnv1a(data: bytes) -> int:
+    h = 0xCBF29CE484222325
+    for b in data:
+        h ^= b
+        h = (h * 0x100000001B3) & 0xFFFFFFFFFFFFFFFF
+    return h
+
+
+def write_container(path, rungs, theta, j_tie, q, tensors) -> None:
+    out = bytearray(_MAGIC)
+    out += _st.pack("<II", 1, len(rungs))
+    for S, k in rungs:
+        out += _st.pack("<ii", S, k)
+    for th in theta:
+        out += _st.pack("<d", th)
+    out += _st.pack("<id", j_tie, q)
+    taps = taps_table()
+    for S in range(8, 17):
+        out += _st.pack("<I", int(taps[S]))
+    out += _st.pack("<I", len(tensors))
+    for t in tensors:
+        name = t.get("name", "").encode()
+        out += _st.pack("<I", len(name)) + name
+        out += _st.pack("<qq", t["rows"], t["cols"])
+        out += np.ascontiguousarray(t["a"], "<f4").tobytes()
+        if t.get("rho") is None:
+            out += _st.pack("<I", 0)
+        else:
+            out += _st.pack("<I", 1) + np.ascontiguousarray(t["rho"], "<f4").tobytes()
+        out += _st.pack("<q", t["tie_count"])
+        cols = np.ascontiguousarray(t.get("outlier_cols", np.zeros(0)), "<i4")
+        out += _st.pack("<i", cols.size) + cols.tobytes()
+        out += np.ascontiguousarray(t.get("outlier_vals", np.zeros(0)), "<u2").tobytes()
+        nbytes = (int(t["stream_bits"]) + 7) // 8
+        out += _st.pack("<QQ", int(t["stream_bits"]), nbytes)
+        out += np.ascontiguousarray(t["stream"], np.uint8)[:nbytes].tobytes()
+    out += _st.pack("<Q", _fnv1a(bytes(out)))
+    with open(path, "wb") as f:
+        f.write(bytes(out))
+
+
+def read_container(path) -> dict:
+    data = open(path, "rb").read()
+    if data[:8] != _MAGIC:
+        raise ValueError("not a container")
+    if _st.unpack("<Q", data[-8:])[0] != _fnv1a(data[:-8]):
+        raise ValueError("hash mismatch")
+    at = 8
+
+    def take(fmt):
+        nonlocal at
+        v = _st.unpack_from(fmt, data, at)
+        at += _st.calcsize(fmt)
+        return v
+
+    version, J = take("<II")
+    if version != 1:
+        raise ValueError("version")
+    rungs = [take("<ii") for _ in range(J)]
+    theta = [take("<d")[0] for _ in range(J - 1)]
+    j_tie, q = take("<id")
+    taps = [take("<I")[0] for _ in range(9)]
+    (nt,) = take("<I")
+    tensors = []
+    for _ in range(nt):
+        (nl,) = take("<I")
+        name = data[at:at + nl].decode()
+        at += nl
+        R, Cc = take("<qq")
+        a = np.frombuffer(data, "<f4", Cc, at).copy()
+        at += 4 * Cc
+        (has_rho,) = take("<I")
+        rho = None
+        if has_rho:
+            rho = np.frombuffer(data, "<f4", R, at).copy()
+            at += 4 * R
+        (T,) = take("<q")
+        (no,) = take("<i")
+        cols = np.frombuffer(data, "<i4", no, at).copy()
+        at += 4 * no
+        vals = np.frombuffer(data, "<u2", R * no, at).copy().reshape(R, no)
+        at += 2 * R * no
+        bits, nbytes = take("<QQ")
+        stream = np.frombuffer(data, np.uint8, nbytes, at).copy()
+        at += nbytes
+        tensors.append({"name": name, "rows": R, "cols": Cc, "a": a, "rho": rho, "tie_count": T,
+                        "outlier_cols": cols, "outlier_vals": vals, "stream": stream,
+                        "stream_bits": bits})
+    if at != len(data) - 8:
+        raise ValueError("trailing bytes")
+    return {"rungs": [tuple(r) for r in rungs], "theta": theta, "j_tie": j_tie, "q": q,
+            "taps": taps, "tensors": tensors}

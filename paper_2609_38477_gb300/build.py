@@ -10,7 +10,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libseedq.so")
-SOURCES = ["plan.cu", "decode.cu", "gemv.cu", "encode.cu"]
+SOURCES = ["plan.cu", "decode.cu", "gemv.cu", "encode.cu", "container.cpp"]
 HEADERS = [os.path.join(CSRC, "seedq_internal.cuh"), os.path.join(ROOT, "include", "seedq.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC"] + ARCH
@@ -34,7 +34,7 @@ def build(force: bool = False, verbose: bool = False) -> str:
     objs, jobs = [], []
     for src in SOURCES:
         s = os.path.join(CSRC, src)
-        o = os.path.join(BUILD, src.replace(".cu", ".o"))
+        o = os.path.join(BUILD, os.path.splitext(src)[0] + ".o")
         objs.append(o)
         if force or _stale(o, [s] + HEADERS):
             jobs.append([nvcc] + FLAGS + ["-c", s, "-o", o])

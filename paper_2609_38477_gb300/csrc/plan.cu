@@ -415,6 +415,8 @@ const char *seedq_status_string(seedq_status s) {
     case SEEDQ_ERR_CUDA: return "CUDA error";
     case SEEDQ_ERR_NOMEM: return "out of memory";
     case SEEDQ_ERR_UNSUPPORTED: return "unsupported rung or shape";
+    case SEEDQ_ERR_IO: return "container file could not be opened, read or written";
+    case SEEDQ_ERR_FORMAT: return "container file is malformed, truncated or corrupted";
   }
   return "unknown status";
 }

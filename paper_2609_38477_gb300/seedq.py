@@ -20,7 +20,7 @@ _lib = None
 
 STATUS = {0: "SEEDQ_OK", 1: "SEEDQ_ERR_INVALID_ARG", 2: "SEEDQ_ERR_STREAM",
           3: "SEEDQ_ERR_SCHEDULE", 4: "SEEDQ_ERR_CUDA", 5: "SEEDQ_ERR_NOMEM",
-          6: "SEEDQ_ERR_UNSUPPORTED"}
+          6: "SEEDQ_ERR_UNSUPPORTED", 7: "SEEDQ_ERR_IO", 8: "SEEDQ_ERR_FORMAT"}
 
 
 class SeedQError(RuntimeError):
@@ -46,6 +46,14 @@ class LayerDesc(C.Structure):
                 ("rho", C.POINTER(C.c_float)), ("tie_count", C.c_int64),
                 ("n_outliers", C.c_int32), ("outlier_cols", C.POINTER(C.c_int32)),
                 ("outlier_vals", C.c_void_p), ("max_batch", C.c_int32)]
+
+
+class ContainerTensor(C.Structure):
+    _fields_ = [("name", C.c_char_p), ("rows", C.c_int64), ("cols", C.c_int64),
+                ("a", C.POINTER(C.c_float)), ("rho", C.POINTER(C.c_float)), ("tie_count", C.c_int64),
+                ("n_outliers", C.c_int32), ("outlier_cols", C.POINTER(C.c_int32)),
+                ("outlier_vals", C.POINTER(C.c_uint16)), ("stream", C.POINTER(C.c_uint8)),
+                ("stream_bits", C.c_uint64)]
 
 
 # Every symbol include/seedq.h declares, with its ctypes signature.
@@ -77,6 +85,13 @@ SIGNATURES = {
                                      C.c_void_p, C.c_void_p]),
     "seedq_pack_stream": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
                                     C.c_uint64, C.c_void_p]),
+    "seedq_container_write": (C.c_int, [C.c_char_p, C.POINTER(Schedule), C.c_int32,
+                                        C.POINTER(ContainerTensor)]),
+    "seedq_container_open": (C.c_int, [C.c_char_p, C.POINTER(C.c_void_p)]),
+    "seedq_container_schedule": (C.c_int, [C.c_void_p, C.POINTER(Schedule)]),
+    "seedq_container_count": (C.c_int, [C.c_void_p, C.POINTER(C.c_int32)]),
+    "seedq_container_get": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(ContainerTensor)]),
+    "seedq_container_close": (C.c_int, [C.c_void_p]),
     "seedq_status_string": (C.c_char_p, [C.c_int]),
     "seedq_last_cuda_error_string": (C.c_char_p, []),
 }
@@ -256,3 +271,106 @@ def encode_blocks(S: int, k: int, w, nblocks: int, seed, E, t, err=None, stream=
     """seedq_encode_blocks: exhaustive seed search of nblocks blocks at rung (S, k)."""
     _check(lib().seedq_encode_blocks(S, k, _ptr(w), nblocks, _ptr(seed), _ptr(E), _ptr(t), _ptr(err),
                                      _stream(stream)), "seedq_encode_blocks")
+
+
+# ------------------------------------------------------------ container
+
+def container_write(path: str, rungs, theta, j_tie: int, q: float, tensors):
+    """seedq_container_write.  tensors: dicts with name, a, rho (or None),
+    tie_count, outlier_cols, outlier_vals (rows x n uint16) and the host
+    stream bytes with its bit length."""
+    rr = (Rung * len(rungs))(*[Rung(int(S), int(k)) for S, k in rungs])
+    th = np.ascontiguousarray(theta if len(theta) else [0.0], np.float64)
+    sched = Schedule(len(rungs), rr, th.ctypes.data_as(C.POINTER(C.c_double)), int(j_tie), float(q))
+    keep, arr = [], (ContainerTensor * max(1, len(tensors)))()
+    for i, t in enumerate(tensors):
+        a = np.ascontiguousarray(t["a"], np.float32)
+        rho = None if t.get("rho") is None else np.ascontiguousarray(t["rho"], np.float32)
+        oc = np.ascontiguousarray(t.get("outlier_cols", np.zeros(0)), np.int32)
+        ov = np.ascontiguousarray(t.get("outlier_vals", np.zeros(0)), np.uint16)
+        st = np.ascontiguousarray(t["stream"], np.uint8)
+        name = t.get("name", "").encode()
+        keep += [a, rho, oc, ov, st, name]
+        arr[i] = ContainerTensor(name, int(t["rows"]), int(t["cols"]),
+                                 a.ctypes.data_as(C.POINTER(C.c_float)),
+                                 None if rho is None else rho.ctypes.data_as(C.POINTER(C.c_float)),
+                                 int(t["tie_count"]), int(oc.size),
+                                 oc.ctypes.data_as(C.POINTER(C.c_int32)),
+                                 ov.ctypes.data_as(C.POINTER(C.c_uint16)),
+                                 st.ctypes.data_as(C.POINTER(C.c_uint8)), int(t["stream_bits"]))
+    _check(lib().seedq_container_write(path.encode(), C.byref(sched), len(tensors), arr),
+           "seedq_container_write")
+
+
+class Container:
+    """seedq_container_open ... seedq_container_close: a read-only view."""
+
+    def __init__(self, path: str):
+        h = C.c_void_p()
+        _check(lib().seedq_container_open(path.encode(), C.byref(h)), "seedq_container_open")
+        self.h = h
+        s = Schedule()
+        _check(lib().seedq_container_schedule(self.h, C.byref(s)), "seedq_container_schedule")
+        self.rungs = [(s.rungs[j].S, s.rungs[j].k) for j in range(s.J)]
+        self.theta = [s.theta[j] for j in range(s.J - 1)]
+        self.j_tie, self.q = s.j_tie, s.q
+        n = C.c_int32()
+        _check(lib().seedq_container_count(self.h, C.byref(n)), "seedq_container_count")
+        self.count = n.value
+
+    def tensor(self, i: int) -> dict:
+        t = ContainerTensor()
+        _check(lib().seedq_container_get(self.h, i, C.byref(t)), "seedq_container_get")
+        R, Cc, no = t.rows, t.cols, t.n_outliers
+        nbytes = (t.stream_bits + 7) // 8
+        return {
+            "name": t.name.decode(), "rows": R, "cols": Cc,
+            "a": np.ctypeslib.as_array(t.a, (Cc,)).copy(),
+            "rho": None if not t.rho else np.ctypeslib.as_array(t.rho, (R,)).copy(),
+            "tie_count": t.tie_count,
+            "outlier_cols": np.ctypeslib.as_array(t.outlier_cols, (no,)).copy() if no else np.zeros(0, np.int32),
+            "outlier_vals": (np.ctypeslib.as_array(t.outlier_vals, (R * no,)).reshape(R, no).copy()
+                             if no else np.zeros((R, 0), np.uint16)),
+            "stream": np.ctypeslib.as_array(t.stream, (nbytes,)).copy() if nbytes else np.zeros(0, np.uint8),
+            "stream_bits": t.stream_bits,
+        }
+
+    def close(self):
+        if self.h is not None and self.h.value:
+            _check(lib().seedq_container_close(self.h), "seedq_container_close")
+        self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def load_layers(path: str, max_batch: int = 1, stream=None):
+    """Open a container and prepare one bound Layer per tensor (streams and
+    outlier values uploaded to the current CUDA device).  Returns a list of
+    (name, Layer)."""
+    import torch
+
+    c = Container(path)
+    out = []
+    try:
+        for i in range(c.count):
+            t = c.tensor(i)
+            ov = None
+            if len(t["outlier_cols"]):
+                ov = torch.from_numpy(t["outlier_vals"].view(np.int16)).cuda()
+            L = Layer(t["rows"], t["cols"], t["a"], t["rho"], c.rungs, c.theta, c.j_tie, c.q,
+                      t["tie_count"], t["outlier_cols"] if len(t["outlier_cols"]) else None, ov,
+                      max_batch=max_batch, stream=stream)
+            L._ovals_keep = ov
+            nbytes = stream_bytes_required(t["stream_bits"])
+            buf = torch.zeros(nbytes, dtype=torch.uint8, device="cuda")
+            if t["stream"].size:
+                buf[:t["stream"].size].copy_(torch.from_numpy(t["stream"]))
+            L.bind_stream(buf, t["stream_bits"], nbytes)
+            out.append((t["name"], L))
+    finally:
+        c.close()
+    return out
