@@ -33,9 +33,10 @@ constexpr int kMaxCtas = 256;
 
 template <int NB>
 struct Cfg {
-  // Columns per stage and row groups per round, sized so 12 warps' double
-  // buffers and the round's partial sums fit in shared memory.
-  static constexpr int ST = NB == 1 ? 24 : NB == 2 ? 16 : NB <= 8 ? 8 : 4;
+  // Columns per stage and row groups per round: the widest stage for which
+  // 12 warps' double buffers, the jump tables and the round's partial sums
+  // fit in shared memory (wider stages amortize staging and bookkeeping).
+  static constexpr int ST = NB == 1 ? 27 : NB == 2 ? 21 : NB == 4 ? 15 : NB == 8 ? 12 : 7;
   static constexpr int RG = NB == 1 ? 8 : NB <= 4 ? 4 : 1;
   // 16-byte pieces per staged row: ST blocks of at most 44 bits, the 96-bit
   // read-ahead of the last block, and up to 15 + 15 bytes of alignment.
