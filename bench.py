@@ -316,8 +316,16 @@ def our_arm(args):
     sched = load_schedule(args.workload)
     n = args.batch
     gts = G.prepare_workload(w, sched, max_batch=n)
-    xs = [G.x_device(w, i, n) for i in range(len(w.tensors))]
-    ys = [torch.empty((n, t.R), dtype=torch.float32, device="cuda") for t in w.tensors]
+    # All activations of a step in one device buffer and all outputs in one
+    # (views per tensor), so a step's inputs and results move in one copy each.
+    xcat = torch.cat([G.x_device(w, i, n).reshape(-1) for i in range(len(w.tensors))])
+    ycat = torch.empty(sum(n * t.R for t in w.tensors), dtype=torch.float32, device="cuda")
+    xs, ys, ox, oy = [], [], 0, 0
+    for t in w.tensors:
+        xs.append(xcat[ox:ox + n * t.C].view(n, t.C))
+        ys.append(ycat[oy:oy + n * t.R].view(n, t.R))
+        ox += n * t.C
+        oy += n * t.R
     flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
     stream = torch.cuda.current_stream()
     h = stream.cuda_stream
@@ -365,21 +373,21 @@ def our_arm(args):
         for i in range(len(gts)):
             per_call[i].append(evs[i].elapsed_time(evs[i + 1]))
 
-    # End to end through the C ABI with host buffers: H2D of x, D2H of y.
-    xh = [x.cpu().pin_memory() for x in xs]
-    yh = [torch.empty(y.shape, dtype=torch.float32).pin_memory() for y in ys]
-    h2d = sum(x.numel() * 2 for x in xs)
-    d2h = sum(y.numel() * 4 for y in ys)
+    # End to end through the C ABI with host buffers: every step copies its
+    # activations in from pinned host memory and its outputs back (one copy
+    # each way), then waits for them on the host.
+    xh = xcat.cpu().pin_memory()
+    yh = torch.empty(ycat.shape, dtype=torch.float32).pin_memory()
+    h2d = xcat.numel() * 2
+    d2h = ycat.numel() * 4
     e2e_ms = []
     for _ in range(args.steps):
         flush.zero_()
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
-        for xd, xhh in zip(xs, xh):
-            xd.copy_(xhh, non_blocking=True)
+        xcat.copy_(xh, non_blocking=True)
         step()
-        for yd, yhh in zip(ys, yh):
-            yhh.copy_(yd, non_blocking=True)
+        yh.copy_(ycat, non_blocking=True)
         b.record(stream)
         b.synchronize()
         e2e_ms.append(a.elapsed_time(b))
