@@ -158,6 +158,12 @@ def dist_max(v: float) -> float:
     return float(t.item())
 
 
+def replica_value(world: int, n: int, slowest_ms: float) -> float:
+    """Whole-job rate of N independent replicas: every rank runs n tokens per
+    step, and the job's step is the slowest rank's."""
+    return world * n / (slowest_ms * 1e-3)
+
+
 def dist_barrier():
     import torch.distributed as dist
 
@@ -406,7 +412,7 @@ def our_arm(args):
     achieved_issue = warp_inst / (kern_ms * 1e-3) / 1e9
     achieved_hbm = alg_bytes / (kern_ms * 1e-3) / 1e9
     stream_bytes = sum((gt.bits + 7) // 8 for gt in gts)
-    value = world * n / (mean_step * 1e-3)
+    value = replica_value(world, n, mean_step)
 
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
