@@ -28,8 +28,9 @@
 // instructions on the IEEE bit patterns instead: integers and exact products
 // are converted to doubles by building their bits, products by powers of two
 // add to the exponent field, and comparisons of magnitudes compare bit
-// patterns.  Only the rounded steps (sums, products and quotients of the
-// solve, the error) run on the fp64 pipe.
+// patterns; the quotients of the solve are exact IEEE divisions done with
+// 64-bit integer arithmetic (div_rn).  Only the rounded sums and products of
+// the solve and the error run on the fp64 pipe.
 #include "seedq_internal.cuh"
 
 namespace seedq {
@@ -159,7 +160,10 @@ __device__ __forceinline__ void search_block(int S, const uint64_t *tab, const f
       }
     }
     // Gaussian elimination with partial pivoting (first row of largest |pivot|).
+    // Divisions are exact IEEE quotients on the integer pipes (div_rn), one
+    // reciprocal estimate per pivot, reused by the back substitution.
     bool singular = false;
+    DivRecip Rp[K];
 #pragma unroll
     for (int c = 0; c < K; ++c) {
       int pr = c;
@@ -187,9 +191,10 @@ __device__ __forceinline__ void search_block(int S, const uint64_t *tab, const f
           b[r] = tb;
         }
       }
+      Rp[c] = div_recip(A[c][c]);
 #pragma unroll
       for (int r = c + 1; r < K; ++r) {
-        const double f = A[r][c] / A[c][c];
+        const double f = div_rn(A[r][c], Rp[c]);
 #pragma unroll
         for (int q = c + 1; q < K; ++q) A[r][q] = __dsub_rn(A[r][q], __dmul_rn(f, A[c][q]));
         b[r] = __dsub_rn(b[r], __dmul_rn(f, b[c]));
@@ -202,7 +207,7 @@ __device__ __forceinline__ void search_block(int S, const uint64_t *tab, const f
       double sacc = b[r];
 #pragma unroll
       for (int q = r + 1; q < K; ++q) sacc = __dsub_rn(sacc, __dmul_rn(A[r][q], x[q]));
-      x[r] = sacc / A[r][r];
+      x[r] = div_rn(sacc, Rp[r]);
     }
     // x = tstar * 2^-(S-1); the mantissa of t_j at exponent E is rint(x_j * 2^(S-1-E)).
     // fits() is monotone in E, so the smallest fitting E is found by stepping

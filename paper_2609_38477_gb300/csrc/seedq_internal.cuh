@@ -316,6 +316,114 @@ __device__ __forceinline__ void reconstruct_rt(uint32_t lo, uint32_t hi, const u
 }
 
 
+// ------------------------------------------------- fp64 division, integer pipes
+//
+// a / b rounded to nearest (IEEE), for b normal and a normal or zero with a
+// normal quotient, computed with 64-bit integer instructions only.  With the
+// significands ma, mb in [2^52, 2^53), the quotient's significand is
+// q = floor(ma * 2^s / mb) for s = 52 (ma >= mb) or 53, rounded up when twice
+// the remainder exceeds mb (binary division never lands exactly halfway).  q
+// comes from an estimate of 2^116 / mb (an fp32 reciprocal refined by two
+// Newton steps in fixed point) and is then corrected against the exact
+// 128-bit remainder, so the estimate only has to be within a few units.
+struct DivRecip {
+  double b;      // the divisor (for the rare operands handled by hardware division)
+  uint64_t d;    // significand of b
+  uint64_t inv;  // ~ 2^116 / d
+  int e;         // unbiased exponent of b
+  uint64_t sign; // sign bit of b
+};
+
+__device__ __forceinline__ void mul128(uint64_t a, uint64_t b, uint64_t &hi, uint64_t &lo) {
+  hi = __umul64hi(a, b);
+  lo = a * b;
+}
+
+__device__ __forceinline__ DivRecip div_recip(double b) {
+  const uint64_t bb = (uint64_t)__double_as_longlong(b);
+  DivRecip r;
+  r.b = b;
+  r.sign = bb >> 63;
+  r.e = (int)((bb >> 52) & 2047) - 1023;
+  r.d = (bb & ((1ull << 52) - 1)) | (1ull << 52);
+  // fp32 estimate of 1/d from d's top 24 bits: d ~ (d >> 29) * 2^29.
+  const float df = __uint_as_float((uint32_t)((r.d >> 29) & 0x7fffffu) | ((uint32_t)(127 + 52) << 23));
+  const uint32_t rb = __float_as_uint(__frcp_rn(df));
+  const int er = (int)(rb >> 23) - 127;             // -53 or -52
+  const uint64_t m = (rb & 0x7fffffu) | 0x800000u;  // 1/d ~ m * 2^(er - 23)
+  const int sh = 116 + er - 23;                      // inv ~ m * 2^sh, sh in {40, 41}
+  uint64_t inv = sh >= 41 ? ~0ull : (m << sh);
+  // Two Newton steps: inv += inv * (2^116 - d * inv) / 2^116.
+#pragma unroll
+  for (int it = 0; it < 2; ++it) {
+    uint64_t phi, plo;
+    mul128(r.d, inv, phi, plo);  // d * inv, around 2^116
+    const uint64_t two116 = 1ull << 52;  // 2^116 as (hi = 2^52, lo = 0)
+    bool neg;
+    uint64_t ehi, elo;
+    if (phi >= two116) {
+      neg = true;
+      elo = plo;
+      ehi = phi - two116;  // d*inv - 2^116
+    } else {
+      neg = false;
+      elo = 0ull - plo;
+      ehi = two116 - phi - (plo != 0 ? 1ull : 0ull);
+    }
+    // correction = inv * e / 2^116, with e >> 52 (e < 2^116).
+    const uint64_t e52 = (ehi << 12) | (elo >> 52);
+    const uint64_t corr = __umul64hi(inv, e52);
+    inv = neg ? inv - corr : inv + corr;
+  }
+  r.inv = inv;
+  return r;
+}
+
+__device__ __forceinline__ double div_rn(double a, const DivRecip &R) {
+  const uint64_t ab = (uint64_t)__double_as_longlong(a);
+  const uint64_t sign = (ab >> 63) ^ R.sign;
+  if ((ab & 0x7fffffffffffffffull) == 0) return __longlong_as_double((long long)(sign << 63));
+  const int ea = (int)((ab >> 52) & 2047) - 1023;
+  const uint64_t ma = (ab & ((1ull << 52) - 1)) | (1ull << 52);
+  const int s = ma >= R.d ? 52 : 53;
+  int e = ea - R.e - (s - 52);
+  // Subnormal or non-finite operands, or a quotient near the end of the
+  // exponent range: hardware division (never taken by the encoder's values).
+  if (ea == -1023 || ea == 1024 || R.e == -1023 || R.e == 1024 || e < -1021 || e > 1022) return a / R.b;
+  // N = ma * 2^s as 128 bits.
+  const uint64_t nhi = ma >> (64 - s), nlo = ma << s;
+  const uint64_t n42 = (nhi << 22) | (nlo >> 42);
+  uint64_t q = __umul64hi(n42, R.inv) >> 10;
+  // Exact remainder N - q * d, then correct q by whole units.
+  uint64_t phi, plo;
+  mul128(q, R.d, phi, plo);
+  long long rhi = (long long)(nhi - phi - (nlo < plo ? 1ull : 0ull));
+  uint64_t rlo = nlo - plo;
+#pragma unroll
+  for (int k = 0; k < 3; ++k) {
+    if (rhi < 0) {  // remainder negative: q too large
+      --q;
+      const uint64_t t = rlo + R.d;
+      rhi += (t < rlo) ? 1 : 0;
+      rlo = t;
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < 3; ++k) {
+    if (rhi > 0 || rlo >= R.d) {  // remainder >= d: q too small
+      ++q;
+      rhi -= (rlo < R.d) ? 1 : 0;
+      rlo -= R.d;
+    }
+  }
+  if (2 * rlo > R.d) ++q;  // round to nearest (no ties)
+  if (q == (1ull << 53)) {
+    q = 1ull << 52;
+    ++e;
+  }
+  return __longlong_as_double((long long)((sign << 63) | ((uint64_t)(e + 1023) << 52) | (q - (1ull << 52))));
+}
+
 __host__ __device__ inline uint64_t stream_bytes_required(uint64_t bits) {
   return ((bits + 7) / 8 + 15) / 16 * 16 + 16;
 }
