@@ -170,6 +170,32 @@ seedq_status seedq_gemm_multi(const seedq_layer *const *layers, int32_t count,
                               const uint16_t *const *X, int32_t n, float *const *Y,
                               void *cuda_stream);
 
+/* ------------------------------------------------------------ layer sets
+ * All tensors of a model (or any group of prepared, bound layers) behind one
+ * launch per call: the per-tensor descriptors and, for every batch size up to
+ * the set's max_batch, the cost-balanced split of all their blocks across the
+ * SMs are built once, in device memory, by seedq_layer_set_create
+ * (synchronous; allocates).  A call then needs no host-side work per tensor.
+ * Activations and outputs live in one buffer each: tensor i reads its
+ * n x C_i bfloat16 block at X + n * col_offsets[i] and writes its n x R_i
+ * float32 block at Y + n * row_offsets[i] (offsets from
+ * seedq_layer_set_layout; col_offsets[count] = sum of C_i, likewise rows).
+ * The set captures each layer's bound stream when it is created: rebinding or
+ * releasing a layer requires releasing the set first.  Calls on a set use the
+ * layers' scratch, so they must not overlap with other calls on those layers. */
+typedef struct seedq_layer_set seedq_layer_set;
+
+/* count: 1..65535 layers, each bound; max_batch of the set = the smallest. */
+seedq_status seedq_layer_set_create(const seedq_layer *const *layers, int32_t count,
+                                    seedq_layer_set **out);
+/* Host arrays of count + 1 entries each (either may be NULL). */
+seedq_status seedq_layer_set_layout(const seedq_layer_set *set, int64_t *col_offsets,
+                                    int64_t *row_offsets);
+/* Y_i = X_i W_hat_i^T for every tensor of the set, n = 1..max_batch. */
+seedq_status seedq_gemm_set(const seedq_layer_set *set, const uint16_t *X, int32_t n, float *Y,
+                            void *cuda_stream);
+seedq_status seedq_layer_set_release(seedq_layer_set *set);
+
 /* Host copy of the rung index (0..J-1) of blocks of rows [row0, row0+nrows):
  * rungs_host receives nrows x (C/8) bytes.  Synchronous. */
 seedq_status seedq_layer_rung_map(const seedq_layer *layer, int64_t row0,

@@ -21,6 +21,11 @@
 // one partial sum per CTA in scratch; the CTA that arrives last adds them in
 // CTA order.  No result depends on timing.
 #include <cuda_fp16.h>
+#include <string.h>
+
+#include <cstddef>
+#include <new>
+#include <vector>
 
 #include "seedq_internal.cuh"
 
@@ -55,8 +60,13 @@ struct TensorArgs {
   float *y;               // n x R
   int64_t ubegin;         // first unit of this tensor in the launch's sequence
   uint64_t stream_bytes;  // readable bytes of the bound stream buffer
+  int64_t cpre, rpre;     // layer sets: columns and rows of the tensors before it
 };
 
+// One launch over several tensors.  The descriptors and the CTA ranges are
+// either inline (seedq_gemm_multi, up to kMaxTensors) or, for a layer set,
+// in device memory, with every tensor's x and y at fixed offsets of one
+// activation and one output buffer.
 struct MultiArgs {
   TensorArgs t[kMaxTensors];
   int nt;
@@ -64,6 +74,10 @@ struct MultiArgs {
   int ctas;
   uint32_t zero;  // 0 at run time; keeps per-rung constants in registers
   int64_t cta_begin[kMaxCtas + 1];
+  const TensorArgs *tens;  // layer set: nt descriptors (else t)
+  const int64_t *cbd;      // layer set: ctas + 1 range starts (else cta_begin)
+  const uint16_t *Xall;    // layer set: x of tensor i at Xall + n * cpre_i
+  float *Yall;             // layer set: y of tensor i at Yall + n * rpre_i
 };
 
 __host__ __device__ inline int batch_template(int n) {
@@ -80,12 +94,12 @@ __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commi
 template <int N>
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
 
-// CTA whose range holds unit u.
-__device__ __forceinline__ int cta_of(const MultiArgs &a, int64_t u) {
-  int lo = 0, hi = a.ctas - 1;
+// CTA whose range holds unit u (cb: the ctas + 1 range starts).
+__device__ __forceinline__ int cta_of(const int64_t *cb, int ctas, int64_t u) {
+  int lo = 0, hi = ctas - 1;
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
-    if (a.cta_begin[mid] <= u) lo = mid;
+    if (cb[mid] <= u) lo = mid;
     else hi = mid - 1;
   }
   return lo;
@@ -383,22 +397,57 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ Mu
   int *flag = reinterpret_cast<int *>(comb + CF::RG * kWarps * 32 * NB);
   {
     // The jump tables depend only on S, so any tensor's copy serves all.
-    const uint4 *src = reinterpret_cast<const uint4 *>(a.t[0].p.tables);
+    const uint4 *src = reinterpret_cast<const uint4 *>((a.tens ? a.tens : a.t)[0].p.tables);
     uint4 *dst = reinterpret_cast<uint4 *>(tabs);
     for (int i = threadIdx.x; i < kTableSlots * 256; i += kThreads) dst[i] = __ldg(src + i);
   }
   // The permuted activations come from the pre-kernel launched just before.
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const int cta = blockIdx.x;
-  const int64_t u0 = a.cta_begin[cta], u1 = a.cta_begin[cta + 1];
+  const TensorArgs *tens = a.tens ? a.tens : a.t;
+  const int64_t *cb = a.cbd ? a.cbd : a.cta_begin;
+  const int64_t u0 = cb[cta], u1 = cb[cta + 1];
   int64_t u = u0;
   bool first = true;
+  // The round's tensor descriptor, copied to shared memory (for a layer set
+  // with its x and y pointers filled in).
+  __shared__ TensorArgs sT;
+  constexpr int kTWords = sizeof(TensorArgs) / 4;
+  static_assert(sizeof(TensorArgs) % 8 == 0, "descriptor size");
+  constexpr int kXWord = offsetof(TensorArgs, x) / 4, kYWord = offsetof(TensorArgs, y) / 4;
+  int ti = 0;
+  {
+    int lo = 0, hi = a.nt - 1;  // last tensor whose first unit is <= u0
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (tens[mid].ubegin <= u0) lo = mid;
+      else hi = mid - 1;
+    }
+    ti = lo;
+  }
   while (u < u1) {
-    int ti = 0;
-    while (ti + 1 < a.nt && a.t[ti + 1].ubegin <= u) ++ti;
-    const TensorArgs &T = a.t[ti];
+    while (ti + 1 < a.nt && tens[ti + 1].ubegin <= u) ++ti;
+    {
+      const uint32_t *srcw = reinterpret_cast<const uint32_t *>(tens + ti);
+      uint32_t *dstw = reinterpret_cast<uint32_t *>(&sT);
+      const uint64_t xv = a.tens ? (uint64_t)(a.Xall + (int64_t)a.n * tens[ti].cpre) : 0;
+      const uint64_t yv = a.tens ? (uint64_t)(a.Yall + (int64_t)a.n * tens[ti].rpre) : 0;
+      for (int w = threadIdx.x; w < kTWords; w += kThreads) {
+        uint32_t v = srcw[w];
+        if (a.tens) {
+          if (w == kXWord) v = (uint32_t)xv;
+          if (w == kXWord + 1) v = (uint32_t)(xv >> 32);
+          if (w == kYWord) v = (uint32_t)yv;
+          if (w == kYWord + 1) v = (uint32_t)(yv >> 32);
+        }
+        dstw[w] = v;
+      }
+    }
+    const TensorArgs &T = sT;
     const LayerArgs &p = T.p;
-    const int64_t tend = (ti + 1 < a.nt) ? a.t[ti + 1].ubegin : a.cta_begin[a.ctas];
+    const int64_t tub = tens[ti].ubegin;
+    const int tnb = tens[ti].p.nb;
+    const int64_t tend = (ti + 1 < a.nt) ? tens[ti + 1].ubegin : cb[a.ctas];
     const int64_t rend = min(u1, tend);
     // The next round: up to RG row groups of this tensor.
     // (In shared memory: the stage issue indexes it by a runtime piece number.)
@@ -407,14 +456,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ Mu
     int np = 0, nst_total = 0;
     int64_t uu = u;
     while (uu < rend && np < CF::RG) {
-      const int64_t lu = uu - T.ubegin;
-      const int64_t g = lu / p.nb;
-      const int ca = (int)(lu - g * p.nb);
-      const int cb = (int)min((int64_t)p.nb, ca + (rend - uu));
-      if (threadIdx.x == 0) pcs[np] = Piece{g, ca, cb};
-      nst_total += (cb - ca + CF::ST - 1) / CF::ST;
+      const int64_t lu = uu - tub;
+      const int64_t g = lu / tnb;
+      const int ca = (int)(lu - g * tnb);
+      const int cbk = (int)min((int64_t)tnb, ca + (rend - uu));
+      if (threadIdx.x == 0) pcs[np] = Piece{g, ca, cbk};
+      nst_total += (cbk - ca + CF::ST - 1) / CF::ST;
       ++np;
-      uu += cb - ca;
+      uu += cbk - ca;
     }
     for (int i = threadIdx.x; i < np * kWarps * 32 * NB; i += kThreads) comb[i] = 0.f;
     __syncthreads();
@@ -442,18 +491,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ Mu
         __syncthreads();
         if (threadIdx.x == 0) {
           __threadfence();
-          const int cf = cta_of(a, gu), cl = cta_of(a, gu + p.nb - 1);
+          const int cf = cta_of(cb, a.ctas, gu), cl = cta_of(cb, a.ctas, gu + p.nb - 1);
           const int old = atomicAdd(p.counters + g, 1);
           *flag = (old == cl - cf) ? 1 : 0;
         }
         __syncthreads();
         if (*flag) {
           __threadfence();
-          const int cf = cta_of(a, gu), cl = cta_of(a, gu + p.nb - 1);
+          const int cf = cta_of(cb, a.ctas, gu), cl = cta_of(cb, a.ctas, gu + p.nb - 1);
           for (int i = threadIdx.x; i < 32 * NB; i += kThreads) {
             float v = 0.f;
             for (int c2 = cf; c2 <= cl; ++c2) {
-              const int s2 = (a.cta_begin[c2] >= gu) ? 0 : 1;
+              const int s2 = (cb[c2] >= gu) ? 0 : 1;
               v += __ldcg(p.slots + ((int64_t)c2 * 2 + s2) * 32 * kMaxBatch + i);
             }
             const int ln = i / NB, b = i - ln * NB;
@@ -510,6 +559,29 @@ __global__ void k_xperm(const __grid_constant__ XpermArgs a) {
   }
 }
 
+// The same for a layer set: descriptors in device memory, x of tensor i at
+// Xall + n * cpre_i.
+__global__ void k_xperm_set(const TensorArgs *__restrict__ tens, const uint16_t *Xall, int n, int nbt) {
+  asm volatile("griddepcontrol.launch_dependents;");
+  const TensorArgs &T = tens[blockIdx.y];
+  const LayerArgs &p = T.p;
+  const uint16_t *x = Xall + (int64_t)n * T.cpre;
+  const int64_t total = (int64_t)nbt * p.C;
+  for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
+       t += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t pc = t / nbt;
+    const int b = (int)(t - pc * nbt);
+    float v = 0.f;
+    if (b < n) {
+      const int col = __ldg(p.perm + pc);
+      bool outl = false;
+      for (int o = 0; o < p.n_out; ++o) outl |= (p.out_cols[o] == col);
+      v = outl ? 0.f : bf16_to_f32(__ldg(x + (int64_t)b * p.C + col));
+    }
+    p.xperm[t] = v;
+  }
+}
+
 template <int NB>
 static size_t smem_bytes() {
   return sizeof(uint64_t) * 512 * kTableSlots + (size_t)kWarps * Cfg<NB>::WARP_BYTES +
@@ -521,7 +593,8 @@ static size_t smem_bytes() {
 // them); inside the group where a range is cut, the first row's rung profile,
 // scaled to the group's cost, places the cut.  One sweep over the groups
 // places all cuts in order.
-static void partition(const seedq_layer *const *layers, int nt, int n, MultiArgs &a) {
+static void partition(const seedq_layer *const *layers, int nt, int n, int64_t *ubegin, int64_t *cta_begin,
+                      int &ctas_out) {
   const double cb = cost_block(n);
   auto gcost = [&](const seedq_layer *L, int64_t g) { return kCostK * L->h_gk[g] + cb * L->h_gp[g]; };
   int64_t U = 0;
@@ -529,16 +602,16 @@ static void partition(const seedq_layer *const *layers, int nt, int n, MultiArgs
   for (int i = 0; i < nt; ++i) {
     const seedq_layer *L = layers[i];
     const int64_t G = (L->args.R + 31) / 32;
-    a.t[i].ubegin = U;
+    ubegin[i] = U;
     U += G * L->args.nb;
     total += gcost(L, G);
   }
   int ctas = layers[0]->max_ctas;
   if (ctas > kMaxCtas) ctas = kMaxCtas;
   if (U < ctas) ctas = (int)U;
-  a.ctas = ctas;
-  a.cta_begin[0] = 0;
-  a.cta_begin[ctas] = U;
+  ctas_out = ctas;
+  cta_begin[0] = 0;
+  cta_begin[ctas] = U;
   int c = 1;
   double tbase = 0.0;  // cost of the tensors before the current one
   for (int ti = 0; ti < nt && c < ctas; ++ti) {
@@ -574,10 +647,10 @@ static void partition(const seedq_layer *const *layers, int nt, int n, MultiArgs
         }
         if (col < 0) col = 0;
         if (col > nb) col = nb;
-        int64_t u = a.t[ti].ubegin + g * nb + col;
-        if (u <= a.cta_begin[c - 1]) u = a.cta_begin[c - 1] + 1;
+        int64_t u = ubegin[ti] + g * nb + col;
+        if (u <= cta_begin[c - 1]) u = cta_begin[c - 1] + 1;
         if (u > U - (ctas - c)) u = U - (ctas - c);
-        a.cta_begin[c] = u;
+        cta_begin[c] = u;
         ++c;
         target = total * c / ctas;
       }
@@ -586,9 +659,9 @@ static void partition(const seedq_layer *const *layers, int nt, int n, MultiArgs
   }
   // Cuts left over by rounding at the very end of the sequence.
   for (; c < ctas; ++c) {
-    int64_t u = a.cta_begin[c - 1] + 1;
+    int64_t u = cta_begin[c - 1] + 1;
     if (u > U - (ctas - c)) u = U - (ctas - c);
-    a.cta_begin[c] = u;
+    cta_begin[c] = u;
   }
 }
 
@@ -606,7 +679,13 @@ static seedq_status launch(const seedq_layer *const *layers, int nt, const uint1
     a->t[i].y = y[i];
     a->t[i].stream_bytes = layers[i]->stream_bytes;
   }
-  partition(layers, nt, n, *a);
+  int64_t ub[kMaxTensors];
+  partition(layers, nt, n, ub, a->cta_begin, a->ctas);
+  for (int i = 0; i < nt; ++i) a->t[i].ubegin = ub[i];
+  a->tens = nullptr;
+  a->cbd = nullptr;
+  a->Xall = nullptr;
+  a->Yall = nullptr;
   static bool attr_set = false;
   seedq_status rc = SEEDQ_OK;
   if (!attr_set) {
@@ -674,9 +753,162 @@ static seedq_status gemm_multi(const seedq_layer *const *layers, int nt, const u
 
 }  // namespace seedq
 
+// Every tensor of a model (or any group of prepared layers) under one launch:
+// descriptors and, per batch template, the cost-balanced CTA ranges live in
+// device memory, built once when the set is created.
+struct seedq_layer_set {
+  int nt = 0;
+  int max_batch = 0;
+  int64_t cols = 0, rows = 0;            // totals: x holds n * cols values, y n * rows
+  std::vector<int64_t> cpre, rpre;       // nt + 1 prefix sums
+  seedq::TensorArgs *d_tens = nullptr;   // nt descriptors
+  int64_t *d_cta[5] = {nullptr, nullptr, nullptr, nullptr, nullptr};  // per batch template
+  int ctas[5] = {0, 0, 0, 0, 0};
+  int64_t maxC = 0;
+};
+
+namespace seedq {
+
+static int tmpl_index(int nb) { return nb <= 1 ? 0 : nb <= 2 ? 1 : nb <= 4 ? 2 : nb <= 8 ? 3 : 4; }
+
+template <int NB>
+static seedq_status launch_set(const seedq_layer_set *S, const uint16_t *X, int n, float *Y,
+                               cudaStream_t st) {
+  static bool attr_set = false;
+  if (!attr_set) {
+    const cudaError_t e = cudaFuncSetAttribute(k_gemv<NB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               (int)smem_bytes<NB>());
+    if (e != cudaSuccess) return cuda_fail(e);
+    attr_set = true;
+  }
+  MultiArgs a;
+  memset(&a, 0, sizeof a);
+  a.nt = S->nt;
+  a.n = n;
+  a.zero = 0u;
+  a.ctas = S->ctas[tmpl_index(NB)];
+  a.tens = S->d_tens;
+  a.cbd = S->d_cta[tmpl_index(NB)];
+  a.Xall = X;
+  a.Yall = Y;
+  const int64_t want = ((int64_t)NB * S->maxC + 255) / 256;
+  const int gx = (int)(want < 64 ? want : 64);
+  k_xperm_set<<<dim3(gx, S->nt), 256, 0, st>>>(S->d_tens, X, n, NB);
+  cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(a.ctas);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem_bytes<NB>();
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, k_gemv<NB>, a);
+  }
+  return e == cudaSuccess ? SEEDQ_OK : cuda_fail(e);
+}
+
+static void free_set(seedq_layer_set *S) {
+  if (!S) return;
+  cudaFree(S->d_tens);
+  for (int i = 0; i < 5; ++i) cudaFree(S->d_cta[i]);
+  delete S;
+}
+
+}  // namespace seedq
+
 using namespace seedq;
 
 extern "C" {
+
+seedq_status seedq_layer_set_create(const seedq_layer *const *layers, int32_t count,
+                                    seedq_layer_set **out) {
+  if (!layers || !out || count < 1 || count > 65535) return SEEDQ_ERR_INVALID_ARG;
+  *out = nullptr;
+  int mb = kMaxBatch;
+  for (int i = 0; i < count; ++i) {
+    if (!layers[i]) return SEEDQ_ERR_INVALID_ARG;
+    if (!layers[i]->args.stream) return SEEDQ_ERR_STREAM;
+    if (layers[i]->max_batch < mb) mb = layers[i]->max_batch;
+  }
+  seedq_layer_set *S = new (std::nothrow) seedq_layer_set;
+  if (!S) return SEEDQ_ERR_NOMEM;
+  S->nt = count;
+  S->max_batch = mb;
+  S->cpre.assign(count + 1, 0);
+  S->rpre.assign(count + 1, 0);
+  for (int i = 0; i < count; ++i) {
+    S->cpre[i + 1] = S->cpre[i] + layers[i]->args.C;
+    S->rpre[i + 1] = S->rpre[i] + layers[i]->args.R;
+    if (layers[i]->args.C > S->maxC) S->maxC = layers[i]->args.C;
+  }
+  S->cols = S->cpre[count];
+  S->rows = S->rpre[count];
+  std::vector<TensorArgs> h(count);
+  std::vector<int64_t> ub(count), cta(kMaxCtas + 1);
+  seedq_status rc = SEEDQ_OK;
+  cudaError_t e = cudaSuccess;
+  for (int k = 0; k < 5 && rc == SEEDQ_OK && e == cudaSuccess; ++k) {
+    const int nb = 1 << k;
+    if (k > 0 && (1 << (k - 1)) >= mb) break;  // templates above max_batch are never launched
+    int ctas = 0;
+    partition(layers, count, nb, ub.data(), cta.data(), ctas);
+    S->ctas[k] = ctas;
+    e = cudaMalloc((void **)&S->d_cta[k], sizeof(int64_t) * (ctas + 1));
+    if (e == cudaSuccess)
+      e = cudaMemcpy(S->d_cta[k], cta.data(), sizeof(int64_t) * (ctas + 1), cudaMemcpyHostToDevice);
+  }
+  for (int i = 0; i < count; ++i) {
+    memset(&h[i], 0, sizeof(TensorArgs));
+    h[i].p = layers[i]->args;
+    h[i].ubegin = ub[i];
+    h[i].stream_bytes = layers[i]->stream_bytes;
+    h[i].cpre = S->cpre[i];
+    h[i].rpre = S->rpre[i];
+  }
+  if (e == cudaSuccess) e = cudaMalloc((void **)&S->d_tens, sizeof(TensorArgs) * count);
+  if (e == cudaSuccess)
+    e = cudaMemcpy(S->d_tens, h.data(), sizeof(TensorArgs) * count, cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) rc = cuda_fail(e);
+  if (rc != SEEDQ_OK) {
+    free_set(S);
+    return rc;
+  }
+  *out = S;
+  return SEEDQ_OK;
+}
+
+seedq_status seedq_layer_set_layout(const seedq_layer_set *S, int64_t *col_offsets,
+                                    int64_t *row_offsets) {
+  if (!S) return SEEDQ_ERR_INVALID_ARG;
+  for (int i = 0; i <= S->nt; ++i) {
+    if (col_offsets) col_offsets[i] = S->cpre[i];
+    if (row_offsets) row_offsets[i] = S->rpre[i];
+  }
+  return SEEDQ_OK;
+}
+
+seedq_status seedq_gemm_set(const seedq_layer_set *S, const uint16_t *X, int32_t n, float *Y,
+                            void *cuda_stream) {
+  if (!S || !X || !Y || n < 1 || n > S->max_batch) return SEEDQ_ERR_INVALID_ARG;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  switch (batch_template(n)) {
+    case 1: return launch_set<1>(S, X, n, Y, st);
+    case 2: return launch_set<2>(S, X, n, Y, st);
+    case 4: return launch_set<4>(S, X, n, Y, st);
+    case 8: return launch_set<8>(S, X, n, Y, st);
+    default: return launch_set<16>(S, X, n, Y, st);
+  }
+}
+
+seedq_status seedq_layer_set_release(seedq_layer_set *S) {
+  if (!S) return SEEDQ_ERR_INVALID_ARG;
+  free_set(S);
+  return SEEDQ_OK;
+}
 
 seedq_status seedq_gemm_small_batch(const seedq_layer *L, const uint16_t *X, int32_t n, float *Y,
                                     void *cuda_stream) {

@@ -92,6 +92,10 @@ SIGNATURES = {
     "seedq_container_count": (C.c_int, [C.c_void_p, C.POINTER(C.c_int32)]),
     "seedq_container_get": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(ContainerTensor)]),
     "seedq_container_close": (C.c_int, [C.c_void_p]),
+    "seedq_layer_set_create": (C.c_int, [C.POINTER(C.c_void_p), C.c_int32, C.POINTER(C.c_void_p)]),
+    "seedq_layer_set_layout": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
+    "seedq_gemm_set": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p]),
+    "seedq_layer_set_release": (C.c_int, [C.c_void_p]),
     "seedq_status_string": (C.c_char_p, [C.c_int]),
     "seedq_last_cuda_error_string": (C.c_char_p, []),
 }
@@ -271,6 +275,36 @@ def encode_blocks(S: int, k: int, w, nblocks: int, seed, E, t, err=None, stream=
     """seedq_encode_blocks: exhaustive seed search of nblocks blocks at rung (S, k)."""
     _check(lib().seedq_encode_blocks(S, k, _ptr(w), nblocks, _ptr(seed), _ptr(E), _ptr(t), _ptr(err),
                                      _stream(stream)), "seedq_encode_blocks")
+
+
+class LayerSet:
+    """seedq_layer_set_create ... _release: every layer of a model behind one
+    launch per call; x / y of all tensors in one buffer each (see layout())."""
+
+    def __init__(self, layers):
+        self.layers = list(layers)  # kept alive with the set
+        arr = (C.c_void_p * len(self.layers))(*[l.h.value for l in self.layers])
+        h = C.c_void_p()
+        _check(lib().seedq_layer_set_create(arr, len(self.layers), C.byref(h)), "seedq_layer_set_create")
+        self.h = h
+        co = np.zeros(len(self.layers) + 1, np.int64)
+        ro = np.zeros(len(self.layers) + 1, np.int64)
+        _check(lib().seedq_layer_set_layout(self.h, co.ctypes.data, ro.ctypes.data), "seedq_layer_set_layout")
+        self.col_offsets, self.row_offsets = co, ro
+
+    def gemm(self, X, n: int, Y, stream=None):
+        _check(lib().seedq_gemm_set(self.h, _ptr(X), n, _ptr(Y), _stream(stream)), "seedq_gemm_set")
+
+    def release(self):
+        if self.h is not None and self.h.value:
+            _check(lib().seedq_layer_set_release(self.h), "seedq_layer_set_release")
+        self.h = None
+
+    def __del__(self):
+        try:
+            self.release()
+        except Exception:
+            pass
 
 
 # ------------------------------------------------------------ container

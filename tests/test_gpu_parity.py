@@ -398,3 +398,68 @@ def test_layer_set_multi_launch(name):
     for g in gts:
         assert g.layer.device_error() == 0
         g.layer.release()
+
+
+@pytest.mark.parametrize("name", ["c1", "c2"])
+def test_layer_set_one_launch(name):
+    """A layer set over all seven tensors: one launch per call, x and y of all
+    tensors in one buffer each.  Same partition and arithmetic as the
+    multi-tensor launch, so the outputs are bit-identical to it; every row is
+    also checked against the oracle, at each batch size."""
+    w = W.WORKLOADS[name]
+    d, s = load(name)
+    nbmax = max(w.batches)
+    gts = [G().bind(G().prepare_tensor(w, i, d, max_batch=nbmax)) for i in range(len(w.tensors))]
+    layers = [g.layer for g in gts]
+    ls = Q().LayerSet(layers)
+    co, ro = ls.col_offsets, ls.row_offsets
+    assert list(np.diff(co)) == [t.C for t in w.tensors] and list(np.diff(ro)) == [t.R for t in w.tensors]
+    xbs = [W.x_bf16(w, i, nbmax) for i in range(len(w.tensors))]
+    ref = [otensor(w, i).synth_gemv(s, d["tie_count"][i], W.payload_key(w, i), xbs[i])
+           for i in range(len(w.tensors))]
+    for n in w.batches:
+        X = torch.from_numpy(np.concatenate([x[:n].reshape(-1) for x in xbs]).view(np.int16)).cuda()
+        Y = torch.full((n * int(ro[-1]),), float("nan"), dtype=torch.float32, device="cuda")
+        ls.gemm(X, n, Y)
+        Ym = [torch.empty((n, t.R), dtype=torch.float32, device="cuda") for t in w.tensors]
+        Q().gemm_multi(layers, [x_dev(x[:n]) for x in xbs], n, Ym)
+        torch.cuda.synchronize()
+        Yh = Y.cpu().numpy()
+        for i, t in enumerate(w.tensors):
+            yi = Yh[n * ro[i]:n * ro[i + 1]].reshape(n, t.R)
+            assert np.array_equal(yi, Ym[i].cpu().numpy()), (name, n, t.name)
+            for b in range(n):
+                check_y(yi[b], ref[i][0][b], ref[i][1][b])
+    with pytest.raises(Q().SeedQError):
+        ls.gemm(X, nbmax + 1, Y)
+    ls.release()
+    for g in gts:
+        assert g.layer.device_error() == 0
+        g.layer.release()
+
+
+def test_layer_set_full_model_sampled():
+    """The Llama-3-8B-shaped set (225 tensors) in one launch per call; sampled
+    rows of every tensor against the oracle."""
+    name = "c3"
+    w = W.WORKLOADS[name]
+    d, s = load(name)
+    gts = [G().bind(G().prepare_tensor(w, i, d, max_batch=1)) for i in range(len(w.tensors))]
+    ls = Q().LayerSet([g.layer for g in gts])
+    ro = ls.row_offsets
+    xbs = [W.x_bf16(w, i, 1) for i in range(len(w.tensors))]
+    X = torch.from_numpy(np.concatenate([x.reshape(-1) for x in xbs]).view(np.int16)).cuda()
+    Y = torch.full((int(ro[-1]),), float("nan"), dtype=torch.float32, device="cuda")
+    ls.gemm(X, 1, Y)
+    torch.cuda.synchronize()
+    Yh = Y.cpu().numpy()
+    assert not np.isnan(Yh).any()
+    rng = np.random.default_rng(4242)
+    for i, t in enumerate(w.tensors):
+        r = int(rng.integers(0, t.R))
+        y64, yabs = otensor(w, i).synth_gemv(s, d["tie_count"][i], W.payload_key(w, i), xbs[i], r0=r, nrows=1)
+        err = abs(float(Yh[ro[i] + r]) - y64[0][0])
+        assert err <= TOL * yabs[0][0] + 1e-30, (t.name, r)
+    ls.release()
+    for g in gts:
+        g.layer.release()
