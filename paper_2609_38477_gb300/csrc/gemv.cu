@@ -382,7 +382,11 @@ __device__ __forceinline__ float outlier_term(const TensorArgs &T, int64_t r, in
   return s;
 }
 
-template <int NB>
+// kSet: descriptors in device memory (a layer set), copied per round into
+// shared memory; otherwise read straight from the parameter block, whose
+// fields the instructions take as constant-bank operands (measurably faster
+// for the per-stage bookkeeping at small stages).
+template <int NB, bool kSet>
 __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ MultiArgs a) {
   using CF = Cfg<NB>;
   extern __shared__ __align__(16) uint64_t smem[];
@@ -397,15 +401,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ Mu
   int *flag = reinterpret_cast<int *>(comb + CF::RG * kWarps * 32 * NB);
   {
     // The jump tables depend only on S, so any tensor's copy serves all.
-    const uint4 *src = reinterpret_cast<const uint4 *>((a.tens ? a.tens : a.t)[0].p.tables);
+    const uint4 *src = reinterpret_cast<const uint4 *>((kSet ? a.tens : a.t)[0].p.tables);
     uint4 *dst = reinterpret_cast<uint4 *>(tabs);
     for (int i = threadIdx.x; i < kTableSlots * 256; i += kThreads) dst[i] = __ldg(src + i);
   }
   // The permuted activations come from the pre-kernel launched just before.
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const int cta = blockIdx.x;
-  const TensorArgs *tens = a.tens ? a.tens : a.t;
-  const int64_t *cb = a.cbd ? a.cbd : a.cta_begin;
+  const TensorArgs *tens = kSet ? a.tens : a.t;
+  const int64_t *cb = kSet ? a.cbd : a.cta_begin;
   const int64_t u0 = cb[cta], u1 = cb[cta + 1];
   int64_t u = u0;
   bool first = true;
@@ -427,23 +431,21 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ Mu
   }
   while (u < u1) {
     while (ti + 1 < a.nt && tens[ti + 1].ubegin <= u) ++ti;
-    {
+    if constexpr (kSet) {
       const uint32_t *srcw = reinterpret_cast<const uint32_t *>(tens + ti);
       uint32_t *dstw = reinterpret_cast<uint32_t *>(&sT);
-      const uint64_t xv = a.tens ? (uint64_t)(a.Xall + (int64_t)a.n * tens[ti].cpre) : 0;
-      const uint64_t yv = a.tens ? (uint64_t)(a.Yall + (int64_t)a.n * tens[ti].rpre) : 0;
+      const uint64_t xv = (uint64_t)(a.Xall + (int64_t)a.n * tens[ti].cpre);
+      const uint64_t yv = (uint64_t)(a.Yall + (int64_t)a.n * tens[ti].rpre);
       for (int w = threadIdx.x; w < kTWords; w += kThreads) {
         uint32_t v = srcw[w];
-        if (a.tens) {
-          if (w == kXWord) v = (uint32_t)xv;
-          if (w == kXWord + 1) v = (uint32_t)(xv >> 32);
-          if (w == kYWord) v = (uint32_t)yv;
-          if (w == kYWord + 1) v = (uint32_t)(yv >> 32);
-        }
+        if (w == kXWord) v = (uint32_t)xv;
+        if (w == kXWord + 1) v = (uint32_t)(xv >> 32);
+        if (w == kYWord) v = (uint32_t)yv;
+        if (w == kYWord + 1) v = (uint32_t)(yv >> 32);
         dstw[w] = v;
       }
     }
-    const TensorArgs &T = sT;
+    const TensorArgs &T = kSet ? sT : a.t[ti];
     const LayerArgs &p = T.p;
     const int64_t tub = tens[ti].ubegin;
     const int tnb = tens[ti].p.nb;
@@ -689,7 +691,7 @@ static seedq_status launch(const seedq_layer *const *layers, int nt, const uint1
   static bool attr_set = false;
   seedq_status rc = SEEDQ_OK;
   if (!attr_set) {
-    const cudaError_t e = cudaFuncSetAttribute(k_gemv<NB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    const cudaError_t e = cudaFuncSetAttribute(k_gemv<NB, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                (int)smem_bytes<NB>());
     if (e != cudaSuccess) rc = cuda_fail(e);
     else attr_set = true;
@@ -727,7 +729,7 @@ static seedq_status launch(const seedq_layer *const *layers, int nt, const uint1
       attr[0].val.programmaticStreamSerializationAllowed = 1;
       cfg.attrs = attr;
       cfg.numAttrs = 1;
-      e = cudaLaunchKernelEx(&cfg, k_gemv<NB>, *a);
+      e = cudaLaunchKernelEx(&cfg, k_gemv<NB, false>, *a);
     }
     if (e != cudaSuccess) rc = cuda_fail(e);
   }
@@ -776,7 +778,7 @@ static seedq_status launch_set(const seedq_layer_set *S, const uint16_t *X, int 
                                cudaStream_t st) {
   static bool attr_set = false;
   if (!attr_set) {
-    const cudaError_t e = cudaFuncSetAttribute(k_gemv<NB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    const cudaError_t e = cudaFuncSetAttribute(k_gemv<NB, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                (int)smem_bytes<NB>());
     if (e != cudaSuccess) return cuda_fail(e);
     attr_set = true;
@@ -806,7 +808,7 @@ static seedq_status launch_set(const seedq_layer_set *S, const uint16_t *X, int 
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, k_gemv<NB>, a);
+    e = cudaLaunchKernelEx(&cfg, k_gemv<NB, true>, a);
   }
   return e == cudaSuccess ? SEEDQ_OK : cuda_fail(e);
 }
