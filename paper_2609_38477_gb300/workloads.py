@@ -257,3 +257,163 @@ def a_rho_checksum(w: Workload) -> str:
         if rho is not None:
             h.update(rho.tobytes())
     return h.hexdigest()[:32]
+
+
+# ---------------------------------------------------------------------------
+# Synthetic FP16 checkpoints for the data-free importance (Sec. 3.2) and the
+# outlier-column rules (Sec. 3.5): Llama-shaped decoders with random weights,
+# RMSNorm gains near one with a few massive channels, and planted super
+# weights.  Every value is integer-exact before its single rounding to FP16,
+# so numpy and a device kernel implementing the same counter-based generator
+# produce the same bits.
+
+_D_W, _D_GAIN, _D_MASSIVE, _D_SUPER = 17, 19, 23, 29
+MODEL_KINDS = ("q", "k", "v", "o", "gate", "up", "down")
+
+
+@dataclasses.dataclass(frozen=True)
+class ModelSpec:
+    name: str
+    n_layers: int
+    d_model: int
+    n_heads: int
+    n_kv_heads: int
+    head_dim: int
+    d_ff: int
+    vocab: int
+    seed: int
+    description: str
+
+    @property
+    def q_dim(self) -> int:
+        return self.n_heads * self.head_dim
+
+    @property
+    def kv_dim(self) -> int:
+        return self.n_kv_heads * self.head_dim
+
+    def shape(self, kind: str):
+        d, f = self.d_model, self.d_ff
+        return {"q": (self.q_dim, d), "k": (self.kv_dim, d), "v": (self.kv_dim, d),
+                "o": (d, self.q_dim), "gate": (f, d), "up": (f, d), "down": (d, f),
+                "lm_head": (self.vocab, d)}[kind]
+
+    def tensor_names(self):
+        return [f"l{l}.{k}" for l in range(self.n_layers) for k in MODEL_KINDS] + ["lm_head"]
+
+    @property
+    def weights(self) -> int:
+        per = sum(self.shape(k)[0] * self.shape(k)[1] for k in MODEL_KINDS)
+        return self.n_layers * per + self.vocab * self.d_model
+
+
+MODELS = {
+    "tiny": ModelSpec("tiny", 2, 256, 4, 2, 64, 640, 300, 31,
+                      "2 layers, d 256, 4 query / 2 key-value heads of 64, d_ff 640, vocab 300"),
+    "tiny_mha": ModelSpec("tiny_mha", 3, 256, 4, 4, 64, 512, 272, 37,
+                          "3 layers, d 256, 4 heads of 64 (no sharing), d_ff 512, vocab 272"),
+    "llama2_7b": ModelSpec("llama2_7b", 32, 4096, 32, 32, 128, 11008, 32000, 41,
+                           "Llama-2-7B-shaped: 32 layers, d 4096, 32 heads of 128, d_ff 11008, "
+                           "vocab 32000, FP16"),
+    "llama3_8b": ModelSpec("llama3_8b", 32, 4096, 32, 8, 128, 14336, 128256, 43,
+                           "Llama-3-8B-shaped: 32 layers, d 4096, 32 query / 8 key-value heads, "
+                           "d_ff 14336, vocab 128256, FP16"),
+}
+
+# Weights: z * m * 2^-e rounded once to FP16, z the centred sum of the four
+# 16-bit fields of one splitmix64 output (|z| < 2^17, sd ~37838), m * 2^-e =
+# 9 * 2^-24 (sd ~0.0203); exact in fp32 before the rounding.
+W_SCALE_M, W_SCALE_E = 9, 24
+GAIN_SCALE_E = 19           # gains 1 + z * 2^-19 (sd ~0.072), exact in fp32
+MASSIVE_GAIN = 24.0         # gain of the massive channels (layers >= 1)
+N_MASSIVE = 1
+SUPER_VALUES = (40.0, -36.0)  # planted super weights (~2000 sd), exact in FP16
+
+
+def _kind_index(kind: str) -> int:
+    return MODEL_KINDS.index(kind) if kind in MODEL_KINDS else 7
+
+
+def weight_key(spec: ModelSpec, layer, kind: str) -> int:
+    return derive_key(spec.seed, _D_W, 0xFFFF if layer is None else layer, _kind_index(kind))
+
+
+def irwin_hall4(key: int, start: int, n: int) -> np.ndarray:
+    """Centred sum of the four 16-bit fields of splitmix64 outputs start..start+n-1."""
+    h = splitmix64_at(key, np.arange(start, start + n, dtype=np.uint64))
+    m = np.uint64(0xFFFF)
+    z = (h & m) + ((h >> np.uint64(16)) & m) + ((h >> np.uint64(32)) & m) + (h >> np.uint64(48))
+    return z.astype(np.int64) - 131070
+
+
+def _fp16_of_exact(v32: np.ndarray) -> np.ndarray:
+    return np.asarray(v32, np.float32).astype(np.float16).view(np.uint16)
+
+
+def synth_weight_rows(spec: ModelSpec, layer, kind: str, r0: int, nrows: int) -> np.ndarray:
+    """Rows [r0, r0 + nrows) of a weight matrix as FP16 bits (nrows x C),
+    planted super weights included."""
+    R, C = spec.shape(kind)
+    z = irwin_hall4(weight_key(spec, layer, kind), r0 * C, nrows * C)
+    v = z.astype(np.float32) * np.float32(W_SCALE_M * 2.0 ** -W_SCALE_E)
+    out = _fp16_of_exact(v).reshape(nrows, C)
+    for (l, k, r, c, bits) in super_weights(spec):
+        if l == layer and k == kind and r0 <= r < r0 + nrows:
+            out[r - r0, c] = bits
+    return out
+
+
+def super_weights(spec: ModelSpec):
+    """Planted super weights: (layer, kind, row, column, FP16 bits) in the
+    down projection of layer 1 (layer 0 for one-layer models)."""
+    l = min(1, spec.n_layers - 1)
+    R, C = spec.shape("down")
+    key = derive_key(spec.seed, _D_SUPER)
+    out = []
+    for i, val in enumerate(SUPER_VALUES):
+        r = int(splitmix64_at(key, 2 * i) % np.uint64(R))
+        c = int(splitmix64_at(key, 2 * i + 1) % np.uint64(C))
+        out.append((l, "down", r, c, int(_fp16_of_exact(np.float32(val)))))
+    return out
+
+
+def massive_channels(spec: ModelSpec) -> np.ndarray:
+    key = derive_key(spec.seed, _D_MASSIVE)
+    return (splitmix64_at(key, np.arange(N_MASSIVE, dtype=np.uint64))
+            % np.uint64(spec.d_model)).astype(np.int64)
+
+
+def synth_gain(spec: ModelSpec, layer, which: str) -> np.ndarray:
+    """RMSNorm gain as FP16 bits: which = "attn" / "mlp" (layer's input norms)
+    or "final" (layer None)."""
+    wi = {"attn": 0, "mlp": 1, "final": 2}[which]
+    key = derive_key(spec.seed, _D_GAIN, 0xFFFF if layer is None else layer, wi)
+    z = irwin_hall4(key, 0, spec.d_model)
+    v = np.float32(1.0) + z.astype(np.float32) * np.float32(2.0 ** -GAIN_SCALE_E)
+    if which != "final" and layer is not None and layer >= 1:
+        v[massive_channels(spec)] = MASSIVE_GAIN
+    return _fp16_of_exact(v)
+
+
+class SynthModel:
+    """Host (numpy) view of a synthetic checkpoint; arrays are drawn on demand."""
+
+    def __init__(self, spec: ModelSpec):
+        self.spec = spec
+
+    def weight(self, layer, kind: str) -> np.ndarray:
+        R, _ = self.spec.shape(kind)
+        return synth_weight_rows(self.spec, layer, kind, 0, R)
+
+    def lm_head(self) -> np.ndarray:
+        return self.weight(None, "lm_head")
+
+    def gain(self, layer, which: str) -> np.ndarray:
+        return synth_gain(self.spec, layer, which)
+
+    def tensor(self, i: int) -> np.ndarray:
+        """Tensor i of the model order (per layer q, k, v, o, gate, up, down; the head)."""
+        n = len(MODEL_KINDS)
+        if i == self.spec.n_layers * n:
+            return self.lm_head()
+        return self.weight(i // n, MODEL_KINDS[i % n])
