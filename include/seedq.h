@@ -337,6 +337,125 @@ seedq_status seedq_row_plan_static(const double *abar, const double *rho, int64_
                                    int64_t tie_count, int32_t *brk, uint64_t *row_off,
                                    uint64_t *summary, void *cuda_stream);
 
+/* ------------------------------------------- data-free importance (Sec. 3.2)
+ * What the encoder computes from an FP16 checkpoint before allocating rungs:
+ * the input-side factor a of every tensor, the output-side factor rho of the
+ * rows that write the residual stream, and the outlier columns (Sec. 3.5).
+ *
+ *   Eq. gamma: a = gamma^2 for q, k, v (gain of the attention input norm),
+ *     gate, up (gain of the MLP input norm) and the head (final norm).
+ *   Eq. prop:  a^(o) = repeat_kv((W_v o W_v) a^(in)) (query head h reads
+ *     key-value head h / (n_heads / n_kv_heads)); a^(down)_c = E[silu(g)^2]
+ *     ((W_up o W_up) a^(in))_c, g ~ N(0, ((W_gate o W_gate) a^(in))_c), the
+ *     expectation by 64-node Gauss-Hermite quadrature.
+ *   Backward proxy (Sec. 3.2 output side, App. A.1): G = (W_head o W_head)^T 1;
+ *     for each layer, last first: rho_down = G; G += (W_gate o W_gate)^T Gh +
+ *     (W_up o W_up)^T Gh with Gh = (W_down o W_down)^T G; rho_o = G;
+ *     G += (W_v o W_v)^T Gv with Gv the sum over the query heads of each
+ *     key-value head of (W_o o W_o)^T G.  Norms are the identity here; rows of
+ *     q, k, v, gate, up and the head have rho = 1.  The stored rho vectors
+ *     are divided by their mean (summed in row order): the proxy's overall
+ *     scale grows by a model-dependent factor per layer and carries no
+ *     information (the plan normalizes both factors to unit mean anyway).
+ *   Outlier statistics (Sec. 3.5, App. A.6): per column of every tensor the
+ *     dynamic range max_i |W_ij| / (median_i |W_ij| + 2^-24) (the median of an
+ *     even count is the mean of the two middle values) and the activation
+ *     ratio a_j / mean(a) (mean summed in column order).
+ *
+ * Weights are FP16 bit patterns, row-major [out][in] (rows = outputs), every
+ * matrix 16-byte aligned with in-dimension a multiple of 32; gains FP16 too.
+ * All weight and table pointers are device pointers. */
+typedef struct {
+  const uint16_t *attn_norm, *mlp_norm;  /* d_model gains */
+  const uint16_t *wq, *wk, *wv, *wo, *wgate, *wup, *wdown;
+} seedq_llama_layer;
+
+typedef struct {
+  int32_t n_layers, d_model, n_heads, n_kv_heads, head_dim, d_ff;
+  int64_t vocab;
+  const seedq_llama_layer *layers; /* host array of n_layers entries */
+  const uint16_t *final_norm;      /* d_model gain of the head's input */
+  const uint16_t *lm_head;         /* vocab x d_model */
+} seedq_llama_model;
+
+/* Outputs.  Tensor order of the model: per layer q, k, v, o, gate, up, down,
+ * then the head; "columns in model order" concatenates every tensor's in-
+ * dimension in that order. */
+typedef struct {
+  float *a_o;        /* n_layers x (n_heads head_dim), float32 (App. A.7)     */
+  float *a_down;     /* n_layers x d_ff                                       */
+  float *rho_o;      /* n_layers x d_model: rho of W_o's rows, unit mean      */
+  float *rho_down;   /* n_layers x d_model: rho of W_down's rows, unit mean   */
+  double *dyn_range; /* optional: columns in model order; the statistic where
+                        it is >= 1e3, else 0                                 */
+  double *act_ratio; /* optional: columns in model order                      */
+} seedq_importance_out;
+
+/* One stored outlier column: tensor index in model order and column. */
+typedef struct {
+  int32_t tensor, column;
+} seedq_outlier;
+
+/* The whole analysis over a resident model: tables into *out, then the
+ * outlier selection of App. A.6 (each rule's candidates, dynamic range >= 1e3
+ * and activation ratio >= 1e2, at most 32 per rule by decreasing statistic,
+ * ties by tensor then column; ranked by the better position in the two lists,
+ * ties by tensor then column) into outliers[0..*n_outliers), at most
+ * max_outliers (the paper stores four).  Synchronous: enqueues on cuda_stream,
+ * waits for it, and allocates and frees device scratch.  Errors:
+ * SEEDQ_ERR_INVALID_ARG (null or misaligned pointers, shapes out of range,
+ * in-dimension not a multiple of 32, n_heads not a multiple of n_kv_heads),
+ * SEEDQ_ERR_NOMEM, SEEDQ_ERR_CUDA. */
+seedq_status seedq_importance(const seedq_llama_model *model, const seedq_importance_out *out,
+                              seedq_outlier *outliers, int32_t max_outliers,
+                              int32_t *n_outliers, void *cuda_stream);
+
+/* Outlier statistics of one matrix (the column pass of seedq_importance
+ * alone): dyn_range as above for its C columns (device, C doubles), and the
+ * column sums of squares weighted by row, col_sq[c] = sum_r W_rc^2 g_r (device,
+ * C doubles; g device R floats, or NULL for all ones; col_sq may be NULL).
+ * W device R x C FP16, 16-byte aligned, C a multiple of 32.  Enqueued, not
+ * waited for. */
+seedq_status seedq_column_stats(const uint16_t *W, int64_t R, int64_t C, const float *g,
+                                double *dyn_range, double *col_sq, void *cuda_stream);
+
+/* Test / benchmark input generator (no paper counterpart): n FP16 values
+ * out[i] = fp16_rn(z_i m 2^-e), z_i the sum of the four 16-bit fields of
+ * splitmix64 output number first + i of state key, minus 131070; m in
+ * 1..63, e in 0..40 (exact in float32 before the rounding).  out device,
+ * 16-byte aligned.  Enqueued, not waited for. */
+seedq_status seedq_synth_fp16(uint64_t key, int64_t first, int64_t n, int32_t m, int32_t e,
+                              uint16_t *out, void *cuda_stream);
+
+/* ------------------------------------------------- allocator (Alg. 1, Sec. 3.4)
+ * The encoder-side allocation over a set of tensors sharing one budget: the
+ * floor q = the m-th smallest raw importance over all blocks, m =
+ * ceil(floor_f N); the multiplier lambda by bisection over its IEEE bit
+ * pattern so that the payload bits with thresholds theta_j = lambda / s_j meet
+ * floor(8 rbar N); the tied group at the critical threshold and its demotion
+ * count, spread over the tensors in tensor order (App. A.5).  Importance is
+ * that of Eq. imp with the plan's fixed-order fp64 factors (App. A.7).
+ *   tensors     host array of count descriptors; a and rho are HOST float32
+ *               arrays (rho NULL = 1 on every row); cols a multiple of 8.
+ *   J, S, k     the hull's rungs in increasing rate (S even 8..16, k 2..6).
+ *   slopes      J - 1 hull slopes s_j (decreasing).
+ *   theta       out, J - 1 thresholds; j_tie, q out; tie_count and
+ *               stream_bits out, count entries each (payload bits per tensor).
+ * Synchronous; allocates.  Errors: SEEDQ_ERR_INVALID_ARG, SEEDQ_ERR_SCHEDULE
+ * (budget infeasible, or more than one tied group straddles the budget),
+ * SEEDQ_ERR_NOMEM, SEEDQ_ERR_CUDA. */
+typedef struct {
+  int64_t rows, cols;
+  const float *a;   /* host, cols */
+  const float *rho; /* host, rows, or NULL */
+} seedq_factor_desc;
+
+seedq_status seedq_allocate(const seedq_factor_desc *tensors, int32_t count, int32_t J,
+                            const int32_t *S, const int32_t *k, const double *slopes,
+                            double rbar, double floor_f, double *theta, int32_t *j_tie,
+                            double *q, int64_t *tie_count, uint64_t *stream_bits,
+                            void *cuda_stream);
+
 const char *seedq_status_string(seedq_status status);
 const char *seedq_last_cuda_error_string(void);
 

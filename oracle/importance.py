@@ -19,7 +19,10 @@ Plain numpy in float64, written from the paper's definitions:
   E[g_in,c^2] = sum_r W_rc^2 E[g_out,r^2]; the rows of W_o and W_down take the
   residual scale they write to as rho; all other rows have rho = 1 (the
   conservative variant of App. A.1).
-* Outlier columns (Sec. 3.5, App. A.8): the dynamic-range rule
+* The stored rho is normalized to unit mean within its tensor (reading: the
+  paper normalizes both factors to unit mean before use, and the raw proxy
+  leaves float32 range on deep models).
+* Outlier columns (Sec. 3.5, App. A.6): the dynamic-range rule
   max_i |W_ij| / (median_i |W_ij| + eps) >= 1e3 and the activation rule
   a_j >= 1e2 times the tensor mean; at most 32 per rule, ranked by the better
   position in the two lists, the first four kept for the whole model.
@@ -45,8 +48,8 @@ GH_NODES = 64          # Gauss-Hermite nodes for E[silu(g)^2] (reading)
 EPS_DR = 2.0 ** -24    # eps of the dynamic-range rule (reading: smallest FP16 step)
 DR_MIN = 1.0e3         # Sec. 3.5 dynamic-range threshold
 ACT_MIN = 1.0e2        # Sec. 3.5 activation threshold (times the tensor mean)
-LIST_MAX = 32          # App. A.8: each rule keeps at most its 32 largest values
-N_OUTLIERS = 4         # App. A.8: the first four candidates are stored
+LIST_MAX = 32          # App. A.6: each rule keeps at most its 32 largest values
+N_OUTLIERS = 4         # App. A.6: the first four candidates are stored
 
 # Tensor order of one layer; the model's tensors are these per layer, then the head.
 KINDS = ("q", "k", "v", "o", "gate", "up", "down")
@@ -126,12 +129,21 @@ def rho_proxy(model) -> list:
     return out
 
 
+def unit_mean(v) -> np.ndarray:
+    """v divided by its mean, the mean summed in index order (the stored rho:
+    only its shape within the tensor matters, Eq. imp and App. A.2)."""
+    v = np.asarray(v, np.float64)
+    return v / (np.cumsum(v)[-1] / v.size)
+
+
 def importance_tables(model) -> list:
     """(name, a, rho) for every tensor of the model in its tensor order (per
     layer q, k, v, o, gate, up, down; then the head), a and rho in float32 as
-    stored (rho None where it is 1 on every row)."""
+    stored (rho None where it is 1 on every row; otherwise normalized to unit
+    mean, which keeps the table in float32 range: the proxy's scale grows by a
+    model-dependent factor per layer)."""
     s = model.spec
-    rho = rho_proxy(model)
+    rho = [(unit_mean(ro), unit_mean(rd)) for ro, rd in rho_proxy(model)]
     out = []
     for l in range(s.n_layers):
         a_attn = a_from_gain(model.gain(l, "attn"))
@@ -185,7 +197,7 @@ def rule_list(stats) -> list:
 
 
 def select_outliers(dr_per_tensor, ratio_per_tensor, n_keep: int = N_OUTLIERS) -> list:
-    """App. A.8: both lists, each candidate ranked by its better position in
+    """App. A.6: both lists, each candidate ranked by its better position in
     them, ties by tensor then column; the first n_keep (tensor, column)."""
     L1 = rule_list([(d, DR_MIN) for d in dr_per_tensor])
     L2 = rule_list([(r, ACT_MIN) for r in ratio_per_tensor])

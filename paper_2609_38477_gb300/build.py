@@ -10,7 +10,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libseedq.so")
-SOURCES = ["plan.cu", "decode.cu", "gemv.cu", "encode.cu", "container.cpp"]
+SOURCES = ["plan.cu", "decode.cu", "gemv.cu", "encode.cu", "importance.cu", "container.cpp"]
 HEADERS = [os.path.join(CSRC, "seedq_internal.cuh"), os.path.join(ROOT, "include", "seedq.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC"] + ARCH

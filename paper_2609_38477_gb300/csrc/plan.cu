@@ -6,7 +6,10 @@
 #include <stdlib.h>
 #include <string.h>
 
+#include <vector>
+
 #include "seedq_internal.cuh"
+#include "synth.cuh"
 
 namespace seedq {
 
@@ -247,12 +250,6 @@ __global__ void k_tables(const int32_t *__restrict__ slot_S, uint64_t *__restric
 }
 
 // Synthetic payload of the workload recipe, one thread per block.
-__device__ __forceinline__ uint64_t splitmix64_at(uint64_t key, uint64_t i) {
-  uint64_t z = key + (i + 1ull) * 0x9E3779B97F4A7C15ull;
-  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
-  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
-  return z ^ (z >> 31);
-}
 
 __global__ void k_synth(const __grid_constant__ LayerArgs p, const int32_t *__restrict__ S_of, const int32_t *__restrict__ K_of,
                         uint64_t key, uint32_t *__restrict__ out) {
@@ -805,4 +802,323 @@ extern "C" seedq_status seedq_row_plan_static(const double *abar, const double *
                              scr->tcnt, row_off, summary);
   SEEDQ_CUDA(cudaGetLastError());
   return SEEDQ_OK;
+}
+
+// ------------------------------------------------------------ allocator
+// Alg. 1 over a set of tensors: every count is an integer summed with atomic
+// adds and every importance the same fp64 product as the plan's, so the
+// bisections take the same steps on any device and agree with a sequential
+// evaluation.
+namespace seedq {
+namespace {
+
+struct AllocTensor {
+  const double *abar;  // nb unit-mean block means (ascending)
+  const double *rho;   // rows unit-mean row factors
+  int64_t R;           // rows of the tensor
+  int64_t row0;        // first evaluated row in the launch's row space
+  int32_t nrows;       // evaluated rows (1 when rho is 1 on every row)
+  int32_t nb;
+};
+
+enum AllocMode { kCountLE = 0, kBits = 1, kVmin = 2, kTied = 3 };
+
+struct AllocArgs {
+  const AllocTensor *t;
+  int32_t nt;
+  int64_t rows;        // evaluated rows over all tensors
+  int32_t mode, J;
+  int32_t L[kMaxJ];
+  double q, v;
+  double th[kMaxJ];
+  unsigned long long *total;      // kCountLE / kBits / kTied: one counter
+  unsigned long long *per_tensor; // kBits / kTied: nt counters
+  unsigned long long *vmin;       // kVmin: J - 1 bit patterns
+};
+
+__global__ void k_alloc_eval(const __grid_constant__ AllocArgs a) {
+  const int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  unsigned long long val = 0;
+  int ti = -1;
+  if (g < a.rows) {
+    int lo = 0, hi = a.nt - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (a.t[mid].row0 <= g) lo = mid;
+      else hi = mid - 1;
+    }
+    ti = lo;
+    const AllocTensor &T = a.t[ti];
+    const double rr = T.rho[g - T.row0];
+    const unsigned long long mult = T.nrows == 1 ? (unsigned long long)T.R : 1ull;
+    if (a.mode == kCountLE) {
+      val = (unsigned long long)first_block(T.abar, rr, -INFINITY, T.nb, a.v, true) * mult;
+    } else if (a.mode == kBits) {
+      unsigned long long rb = (unsigned long long)a.L[0] * (unsigned long long)T.nb;
+      for (int j = 0; j < a.J - 1; ++j) {
+        const int n_ge = T.nb - first_block(T.abar, rr, a.q, T.nb, a.th[j], false);
+        rb += (unsigned long long)(a.L[j + 1] - a.L[j]) * (unsigned long long)n_ge;
+      }
+      val = rb * mult;
+    } else if (a.mode == kTied) {
+      val = (unsigned long long)(first_block(T.abar, rr, a.q, T.nb, a.v, true) -
+                                 first_block(T.abar, rr, a.q, T.nb, a.v, false)) * mult;
+    } else {
+      for (int j = 0; j < a.J - 1; ++j) {
+        const int c = first_block(T.abar, rr, a.q, T.nb, a.th[j], false);
+        if (c < T.nb) atomicMin(a.vmin + j, (unsigned long long)__double_as_longlong(imp_at(T.abar, rr, a.q, c)));
+      }
+    }
+  }
+  if (a.mode == kVmin) return;
+  if (val && a.per_tensor) atomicAdd(a.per_tensor + ti, val);
+  for (int o = 16; o > 0; o >>= 1) val += __shfl_xor_sync(0xffffffffu, val, o);
+  if ((threadIdx.x & 31) == 0 && val) atomicAdd(a.total, val);
+}
+
+double from_bits(int64_t p) {
+  double d;
+  memcpy(&d, &p, sizeof d);
+  return d;
+}
+
+int64_t to_bits(double d) {
+  int64_t p;
+  memcpy(&p, &d, sizeof p);
+  return p;
+}
+
+struct Allocator {
+  AllocArgs base;
+  cudaStream_t st;
+  unsigned long long *dev;  // 1 + nt + kMaxJ counters
+  int nt;
+  seedq_status err = SEEDQ_OK;
+
+  // One evaluation: returns the total; per-tensor counts into pt when given.
+  uint64_t run(int mode, double q, double v, const double *th, uint64_t *pt = nullptr,
+               double *vmin = nullptr) {
+    if (err != SEEDQ_OK) return 0;
+    AllocArgs a = base;
+    a.mode = mode;
+    a.q = q;
+    a.v = v;
+    for (int j = 0; j < kMaxJ; ++j) a.th[j] = (th && j + 1 < a.J) ? th[j] : 0.0;
+    a.total = dev;
+    a.per_tensor = pt ? dev + 1 : nullptr;
+    a.vmin = dev + 1 + nt;
+    std::vector<unsigned long long> init(1 + nt + kMaxJ, 0ull);
+    for (int j = 0; j < kMaxJ; ++j) init[1 + nt + j] = (unsigned long long)to_bits(INFINITY);
+    cudaError_t e = cudaMemcpyAsync(dev, init.data(), sizeof(unsigned long long) * init.size(),
+                                    cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess) {
+      const int64_t blocks = (a.rows + 255) / 256;
+      k_alloc_eval<<<(int)blocks, 256, 0, st>>>(a);
+      e = cudaGetLastError();
+    }
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(init.data(), dev, sizeof(unsigned long long) * init.size(),
+                          cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) {
+      err = cuda_fail(e);
+      return 0;
+    }
+    if (pt)
+      for (int t = 0; t < nt; ++t) pt[t] = init[1 + t];
+    if (vmin)
+      for (int j = 0; j + 1 < a.J; ++j) vmin[j] = from_bits((int64_t)init[1 + nt + j]);
+    return init[0];
+  }
+};
+
+}  // namespace
+}  // namespace seedq
+
+extern "C" seedq_status seedq_allocate(const seedq_factor_desc *tensors, int32_t count, int32_t J,
+                                       const int32_t *S, const int32_t *k, const double *slopes,
+                                       double rbar, double floor_f, double *theta, int32_t *j_tie,
+                                       double *q_out, int64_t *tie_count, uint64_t *stream_bits,
+                                       void *cuda_stream) {
+  if (!tensors || count < 1 || count > (1 << 20) || J < 1 || J > kMaxJ || !S || !k ||
+      (J > 1 && (!slopes || !theta)) || !j_tie || !q_out || !tie_count || !stream_bits)
+    return SEEDQ_ERR_INVALID_ARG;
+  if (!(rbar > 0.0) || !(floor_f >= 0.0) || !(floor_f <= 1.0)) return SEEDQ_ERR_INVALID_ARG;
+  int32_t L[kMaxJ] = {0};
+  for (int j = 0; j < J; ++j) {
+    if (!rung_supported(S[j], k[j])) return SEEDQ_ERR_UNSUPPORTED;
+    L[j] = S[j] + 4 * k[j] + 4;
+    if (j > 0 && L[j] <= L[j - 1]) return SEEDQ_ERR_SCHEDULE;
+  }
+  for (int j = 0; j + 1 < J; ++j)
+    if (!(slopes[j] > 0.0) || !isfinite(slopes[j])) return SEEDQ_ERR_SCHEDULE;
+  uint64_t nblocks = 0;
+  for (int t = 0; t < count; ++t) {
+    const seedq_factor_desc &d = tensors[t];
+    if (d.rows < 1 || d.rows > (1ll << 24) || d.cols < 8 || d.cols % 8 || d.cols > kMaxCols || !d.a)
+      return SEEDQ_ERR_INVALID_ARG;
+    double asum = 0.0;
+    for (int64_t c = 0; c < d.cols; ++c) {
+      if (!isfinite(d.a[c]) || d.a[c] < 0.f) return SEEDQ_ERR_INVALID_ARG;
+      asum += d.a[c];
+    }
+    if (!(asum > 0.0)) return SEEDQ_ERR_INVALID_ARG;
+    if (d.rho)
+      for (int64_t r = 0; r < d.rows; ++r)
+        if (!isfinite(d.rho[r]) || !(d.rho[r] > 0.f)) return SEEDQ_ERR_INVALID_ARG;
+    nblocks += (uint64_t)d.rows * (uint64_t)(d.cols / 8);
+  }
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+
+  // Factors of every tensor, exactly as the plan computes them.
+  std::vector<void *> owned;
+  auto cleanup = [&]() {
+    for (void *p : owned) cudaFree(p);
+  };
+  auto dalloc = [&](size_t bytes) -> void * {
+    void *p = nullptr;
+    if (cudaMalloc(&p, bytes) != cudaSuccess) {
+      cudaGetLastError();
+      return nullptr;
+    }
+    owned.push_back(p);
+    return p;
+  };
+  std::vector<AllocTensor> ht(count);
+  int64_t rows_total = 0;
+  for (int t = 0; t < count; ++t) {
+    const seedq_factor_desc &d = tensors[t];
+    const int64_t R = d.rows, C = d.cols;
+    const int nb = (int)(C / 8);
+    float *a_in = (float *)dalloc(sizeof(float) * C);
+    float *rho_in = d.rho ? (float *)dalloc(sizeof(float) * R) : nullptr;
+    int32_t *perm = (int32_t *)dalloc(sizeof(int32_t) * C);
+    double *abar = (double *)dalloc(sizeof(double) * nb);
+    double *rho = (double *)dalloc(sizeof(double) * R);
+    if (!a_in || (d.rho && !rho_in) || !perm || !abar || !rho) {
+      cleanup();
+      return SEEDQ_ERR_NOMEM;
+    }
+    cudaError_t e = cudaMemcpyAsync(a_in, d.a, sizeof(float) * C, cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess && d.rho)
+      e = cudaMemcpyAsync(rho_in, d.rho, sizeof(float) * R, cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess) {
+      k_perm<<<(int)((C + 255) / 256), 256, 0, st>>>(a_in, (int)C, perm);
+      k_abar<<<1, 1024, 0, st>>>(a_in, perm, nb, abar);
+      k_rho<<<1, 1024, 0, st>>>(rho_in, R, rho);
+      e = cudaGetLastError();
+    }
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);  // host inputs may go out of scope
+    if (e != cudaSuccess) {
+      cleanup();
+      return cuda_fail(e);
+    }
+    ht[t] = AllocTensor{abar, rho, R, rows_total, d.rho ? (int32_t)R : 1, nb};
+    rows_total += ht[t].nrows;
+  }
+  AllocTensor *dt = (AllocTensor *)dalloc(sizeof(AllocTensor) * count);
+  unsigned long long *dev = (unsigned long long *)dalloc(sizeof(unsigned long long) * (1 + count + kMaxJ));
+  if (!dt || !dev) {
+    cleanup();
+    return SEEDQ_ERR_NOMEM;
+  }
+  {
+    const cudaError_t e =
+        cudaMemcpyAsync(dt, ht.data(), sizeof(AllocTensor) * count, cudaMemcpyHostToDevice, st);
+    if (e != cudaSuccess) {
+      cleanup();
+      return cuda_fail(e);
+    }
+  }
+  Allocator A;
+  memset(&A.base, 0, sizeof A.base);
+  A.base.t = dt;
+  A.base.nt = count;
+  A.base.rows = rows_total;
+  A.base.J = J;
+  for (int j = 0; j < J; ++j) A.base.L[j] = L[j];
+  A.st = st;
+  A.dev = dev;
+  A.nt = count;
+  auto thresholds = [&](double lambda, double *th) {
+    for (int j = 0; j + 1 < J; ++j) th[j] = lambda / slopes[j];
+  };
+  auto finish = [&](seedq_status rc) {
+    cleanup();
+    return A.err != SEEDQ_OK ? A.err : rc;
+  };
+
+  // Floor: the m-th smallest raw importance, m = ceil(f N) (positive doubles
+  // order as their bit patterns).
+  uint64_t m = (uint64_t)ceil(floor_f * (double)nblocks);
+  if (m < 1) m = 1;
+  int64_t lo = 0, hi = to_bits(INFINITY);
+  while (lo < hi && A.err == SEEDQ_OK) {
+    const int64_t mid = lo + (hi - lo) / 2;
+    if (A.run(kCountLE, 0.0, from_bits(mid), nullptr) >= m) hi = mid;
+    else lo = mid + 1;
+  }
+  const double q = from_bits(lo);
+  *q_out = q;
+
+  // Multiplier: bisection on lambda for payload bits <= floor(8 rbar N).
+  const uint64_t budget = (uint64_t)floor(8.0 * rbar * (double)nblocks);
+  double th_lo[kMaxJ] = {0}, th_hi[kMaxJ] = {0};
+  std::vector<uint64_t> pt(count);
+  thresholds(INFINITY, th_hi);
+  if (A.run(kBits, q, 0.0, th_hi) > budget) return finish(SEEDQ_ERR_SCHEDULE);
+  thresholds(0.0, th_lo);
+  if (A.run(kBits, q, 0.0, th_lo, pt.data()) <= budget) {  // every block on the top rung
+    for (int j = 0; j + 1 < J; ++j) theta[j] = th_lo[j];
+    *j_tie = -1;
+    for (int t = 0; t < count; ++t) {
+      tie_count[t] = 0;
+      stream_bits[t] = pt[t];
+    }
+    return finish(SEEDQ_OK);
+  }
+  lo = 0;
+  hi = to_bits(INFINITY);
+  while (hi - lo > 1 && A.err == SEEDQ_OK) {  // bits(lo) > budget >= bits(hi)
+    const int64_t mid = lo + (hi - lo) / 2;
+    double th[kMaxJ];
+    thresholds(from_bits(mid), th);
+    if (A.run(kBits, q, 0.0, th) > budget) lo = mid;
+    else hi = mid;
+  }
+  thresholds(from_bits(lo), th_lo);
+  thresholds(from_bits(hi), th_hi);
+
+  // The critical tied group: blocks with th_lo[j] <= imp < th_hi[j].
+  double vmin[kMaxJ];
+  A.run(kVmin, q, 0.0, th_lo, nullptr, vmin);
+  int jt = -1;
+  double v = 0.0;
+  for (int j = 0; j + 1 < J; ++j) {
+    if (vmin[j] < th_hi[j]) {
+      if (jt >= 0) return finish(SEEDQ_ERR_SCHEDULE);
+      jt = j;
+      v = vmin[j];
+    }
+  }
+  if (jt < 0) return finish(SEEDQ_ERR_SCHEDULE);
+  for (int j = 0; j + 1 < J; ++j) theta[j] = th_hi[j];
+  theta[jt] = v;
+  const uint64_t b_hi = A.run(kBits, q, 0.0, theta, pt.data());
+  const uint64_t step = (uint64_t)(L[jt + 1] - L[jt]);
+  const uint64_t excess = b_hi > budget ? b_hi - budget : 0;
+  uint64_t T = (excess + step - 1) / step;
+  // App. A.5: demote members of the group in block order (tensor order, then
+  // row-major within a tensor) until the budget is met.
+  std::vector<uint64_t> tied(count, 0);
+  if (T) A.run(kTied, q, v, nullptr, tied.data());
+  for (int t = 0; t < count; ++t) {
+    const uint64_t d = T < tied[t] ? T : tied[t];
+    tie_count[t] = (int64_t)d;
+    T -= d;
+    stream_bits[t] = pt[t] - d * step;
+  }
+  if (T != 0) return finish(SEEDQ_ERR_SCHEDULE);
+  *j_tie = jt;
+  return finish(SEEDQ_OK);
 }

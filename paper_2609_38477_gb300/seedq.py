@@ -56,6 +56,33 @@ class ContainerTensor(C.Structure):
                 ("stream_bits", C.c_uint64)]
 
 
+class LlamaLayer(C.Structure):
+    _fields_ = [("attn_norm", C.c_void_p), ("mlp_norm", C.c_void_p), ("wq", C.c_void_p),
+                ("wk", C.c_void_p), ("wv", C.c_void_p), ("wo", C.c_void_p), ("wgate", C.c_void_p),
+                ("wup", C.c_void_p), ("wdown", C.c_void_p)]
+
+
+class LlamaModel(C.Structure):
+    _fields_ = [("n_layers", C.c_int32), ("d_model", C.c_int32), ("n_heads", C.c_int32),
+                ("n_kv_heads", C.c_int32), ("head_dim", C.c_int32), ("d_ff", C.c_int32),
+                ("vocab", C.c_int64), ("layers", C.POINTER(LlamaLayer)),
+                ("final_norm", C.c_void_p), ("lm_head", C.c_void_p)]
+
+
+class ImportanceOut(C.Structure):
+    _fields_ = [("a_o", C.c_void_p), ("a_down", C.c_void_p), ("rho_o", C.c_void_p),
+                ("rho_down", C.c_void_p), ("dyn_range", C.c_void_p), ("act_ratio", C.c_void_p)]
+
+
+class Outlier(C.Structure):
+    _fields_ = [("tensor", C.c_int32), ("column", C.c_int32)]
+
+
+class FactorDesc(C.Structure):
+    _fields_ = [("rows", C.c_int64), ("cols", C.c_int64), ("a", C.POINTER(C.c_float)),
+                ("rho", C.POINTER(C.c_float))]
+
+
 # Every symbol include/seedq.h declares, with its ctypes signature.
 SIGNATURES = {
     "seedq_layer_prepare": (C.c_int, [C.POINTER(LayerDesc), C.POINTER(Schedule), C.c_void_p,
@@ -96,6 +123,16 @@ SIGNATURES = {
     "seedq_layer_set_layout": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
     "seedq_gemm_set": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p]),
     "seedq_layer_set_release": (C.c_int, [C.c_void_p]),
+    "seedq_importance": (C.c_int, [C.POINTER(LlamaModel), C.POINTER(ImportanceOut),
+                                   C.POINTER(Outlier), C.c_int32, C.POINTER(C.c_int32), C.c_void_p]),
+    "seedq_column_stats": (C.c_int, [C.c_void_p, C.c_int64, C.c_int64, C.c_void_p, C.c_void_p,
+                                     C.c_void_p, C.c_void_p]),
+    "seedq_synth_fp16": (C.c_int, [C.c_uint64, C.c_int64, C.c_int64, C.c_int32, C.c_int32,
+                                   C.c_void_p, C.c_void_p]),
+    "seedq_allocate": (C.c_int, [C.POINTER(FactorDesc), C.c_int32, C.c_int32, C.c_void_p,
+                                 C.c_void_p, C.c_void_p, C.c_double, C.c_double, C.c_void_p,
+                                 C.POINTER(C.c_int32), C.POINTER(C.c_double), C.c_void_p,
+                                 C.c_void_p, C.c_void_p]),
     "seedq_status_string": (C.c_char_p, [C.c_int]),
     "seedq_last_cuda_error_string": (C.c_char_p, []),
 }
@@ -275,6 +312,70 @@ def encode_blocks(S: int, k: int, w, nblocks: int, seed, E, t, err=None, stream=
     """seedq_encode_blocks: exhaustive seed search of nblocks blocks at rung (S, k)."""
     _check(lib().seedq_encode_blocks(S, k, _ptr(w), nblocks, _ptr(seed), _ptr(E), _ptr(t), _ptr(err),
                                      _stream(stream)), "seedq_encode_blocks")
+
+
+def synth_fp16(key: int, first: int, n: int, m: int, e: int, out, stream=None):
+    """seedq_synth_fp16: n generated FP16 values into a device buffer."""
+    _check(lib().seedq_synth_fp16(key & ((1 << 64) - 1), first, n, m, e, _ptr(out), _stream(stream)),
+           "seedq_synth_fp16")
+
+
+def column_stats(W, R: int, Cc: int, dyn_range, g=None, col_sq=None, stream=None):
+    """seedq_column_stats: dynamic-range statistic (and weighted column sums of squares)."""
+    _check(lib().seedq_column_stats(_ptr(W), R, Cc, _ptr(g), _ptr(dyn_range), _ptr(col_sq),
+                                    _stream(stream)), "seedq_column_stats")
+
+
+def importance(dims: dict, layers, final_norm, lm_head, out: dict, max_outliers: int = 4,
+               stream=None):
+    """seedq_importance over a resident FP16 model.
+
+    dims: n_layers, d_model, n_heads, n_kv_heads, head_dim, d_ff, vocab.
+    layers: per layer a dict of device buffers attn_norm, mlp_norm, wq, wk, wv,
+    wo, wgate, wup, wdown.  out: device buffers a_o, a_down, rho_o, rho_down
+    and optionally dyn_range, act_ratio.  Returns the outlier (tensor, column)
+    pairs."""
+    L = len(layers)
+    arr = (LlamaLayer * L)(*[LlamaLayer(*[_ptr(y[k]) for k in (
+        "attn_norm", "mlp_norm", "wq", "wk", "wv", "wo", "wgate", "wup", "wdown")]) for y in layers])
+    m = LlamaModel(dims["n_layers"], dims["d_model"], dims["n_heads"], dims["n_kv_heads"],
+                   dims["head_dim"], dims["d_ff"], dims["vocab"], arr, _ptr(final_norm), _ptr(lm_head))
+    o = ImportanceOut(_ptr(out["a_o"]), _ptr(out["a_down"]), _ptr(out["rho_o"]), _ptr(out["rho_down"]),
+                      _ptr(out.get("dyn_range")), _ptr(out.get("act_ratio")))
+    res = (Outlier * max(max_outliers, 1))()
+    n = C.c_int32(0)
+    _check(lib().seedq_importance(C.byref(m), C.byref(o), res, max_outliers, C.byref(n),
+                                  _stream(stream)), "seedq_importance")
+    return [(res[i].tensor, res[i].column) for i in range(n.value)]
+
+
+def allocate(factors, rungs, slopes, rbar: float, floor_f: float, stream=None):
+    """seedq_allocate: Alg. 1's floor, multiplier bisection and tie pass over
+    a list of (rows, cols, a, rho or None) host arrays.  Returns
+    (theta, j_tie, q, tie_count, stream_bits)."""
+    keep = []
+    descs = (FactorDesc * len(factors))()
+    for i, (R, Cc, a, rho) in enumerate(factors):
+        a32 = np.ascontiguousarray(a, np.float32)
+        keep.append(a32)
+        rp = None
+        if rho is not None:
+            r32 = np.ascontiguousarray(rho, np.float32)
+            keep.append(r32)
+            rp = r32.ctypes.data_as(C.POINTER(C.c_float))
+        descs[i] = FactorDesc(R, Cc, a32.ctypes.data_as(C.POINTER(C.c_float)), rp)
+    J = len(rungs)
+    S = np.asarray([r[0] for r in rungs], np.int32)
+    k = np.asarray([r[1] for r in rungs], np.int32)
+    sl = np.ascontiguousarray(slopes if len(slopes) else [1.0], np.float64)
+    theta = np.zeros(max(J - 1, 1), np.float64)
+    jt, q = C.c_int32(), C.c_double()
+    T = np.zeros(len(factors), np.int64)
+    bits = np.zeros(len(factors), np.uint64)
+    _check(lib().seedq_allocate(descs, len(factors), J, S.ctypes.data, k.ctypes.data, sl.ctypes.data,
+                                rbar, floor_f, theta.ctypes.data, C.byref(jt), C.byref(q),
+                                T.ctypes.data, bits.ctypes.data, _stream(stream)), "seedq_allocate")
+    return theta[:J - 1], jt.value, q.value, T, bits
 
 
 class LayerSet:

@@ -27,7 +27,7 @@ def Q():
 def _declared_symbols():
     txt = open(os.path.join(ROOT, "include", "seedq.h")).read()
     txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
-    return sorted(set(re.findall(r"\b(seedq_[a-z_]+)\s*\(", txt)))
+    return sorted(set(re.findall(r"\b(seedq_[a-z_0-9]+)\s*\(", txt)))
 
 
 def test_every_declared_symbol_is_exported(Q):

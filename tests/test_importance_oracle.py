@@ -177,6 +177,17 @@ def test_rho_proxy_sums_query_heads_sharing_a_value_head():
     assert np.array_equal(out[0][1], after)
 
 
+def test_stored_rho_is_the_proxy_at_unit_mean():
+    m = W.SynthModel(W.MODELS["tiny"])
+    raw = I.rho_proxy(m)
+    tables = I.importance_tables(m)
+    for l, (ro, rd) in enumerate(raw):
+        for got, want in ((tables[7 * l + 3][2], ro), (tables[7 * l + 6][2], rd)):
+            assert got.dtype == np.float32
+            assert np.allclose(got, want / want.mean(), rtol=1e-6)
+            assert abs(float(np.mean(got.astype(np.float64))) - 1.0) < 1e-6
+
+
 # ------------------------------------------------------- outlier rules
 
 @pytest.mark.parametrize("R", [7, 8])
