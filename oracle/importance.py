@@ -37,7 +37,8 @@ the residual connection adds the branch's gradient scale to the stream's; the
 attention back-map sums the query heads that share a key-value head; the median
 of an even count is the mean of the two middle values; eps is the smallest
 positive FP16 number; the activation statistic is a_j divided by the tensor
-mean, the mean summed in column order; ties in the merged ranking fall to the
+mean, the mean the correctly rounded sum over the columns divided by their
+count; ties in the merged ranking fall to the
 tensor index, then the column index.
 """
 from __future__ import annotations
@@ -178,9 +179,12 @@ def dynamic_range(W_bits) -> np.ndarray:
 
 
 def activation_ratio(a) -> np.ndarray:
-    """a_j divided by the tensor mean of a (mean summed in column order)."""
+    """a_j divided by the tensor mean of a; the mean is the correctly rounded
+    sum of a (math.fsum) divided by the column count."""
+    import math
+
     a64 = np.asarray(a, np.float32).astype(np.float64)
-    mean = np.cumsum(a64)[-1] / a64.size
+    mean = math.fsum(a64.tolist()) / a64.size
     return a64 / mean
 
 

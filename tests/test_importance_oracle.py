@@ -219,11 +219,19 @@ def test_thresholds_are_inclusive_and_lists_capped_at_32():
     assert got == [(0, c) for c in range(32)]
 
 
-def test_activation_mean_is_summed_in_column_order():
+def test_activation_mean_is_the_correctly_rounded_sum():
+    from fractions import Fraction
+
     a = np.array([2.0 ** 53, 1.0, 1.0, 1.0], np.float32)
-    # In column order every + 1 rounds back to 2^53 (ties to even); the exact
-    # sum 2^53 + 3 would round to 2^53 + 4.
-    assert I.activation_ratio(a)[1] == 4.0 / 2.0 ** 53
+    # Exact sum 2^53 + 3 lies halfway between two doubles and rounds to even,
+    # 2^53 + 4; summing in column order would give 2^53.
+    exact = sum(Fraction(float(x)) for x in a)
+    assert float(exact) == 2.0 ** 53 + 4
+    assert I.activation_ratio(a)[1] == 1.0 / ((2.0 ** 53 + 4) / 4)
+    rng = np.random.default_rng(9)
+    b = np.exp(rng.normal(0, 6, 1000)).astype(np.float32)
+    mean = float(sum(Fraction(float(x)) for x in b)) / b.size
+    assert np.array_equal(I.activation_ratio(b), b.astype(np.float64) / mean)
 
 
 def test_tiny_model_recovers_planted_super_weights_and_massive_channel():
