@@ -38,14 +38,16 @@ def parse():
     p.add_argument("--workload", default="c1")
     p.add_argument("--batch", type=int, default=1)
     p.add_argument("--no-cpu-baseline", action="store_true")
-    p.add_argument("--path", choices=["gemv", "encode"], default="gemv",
+    p.add_argument("--path", choices=["gemv", "encode", "importance"], default="gemv",
                    help="gemv: the fused decode + GEMV step (default); encode: the exhaustive "
                         "seed-search encoder")
     p.add_argument("--rung", default="16,3", help="encoder rung S,k")
     p.add_argument("--blocks", type=int, default=4864, help="encoder blocks per step")
+    p.add_argument("--model", default="llama2_7b",
+                   help="synthetic FP16 checkpoint of the importance path")
     a = p.parse_args()
     if a.steps is None:
-        a.steps = 2000 if a.path == "gemv" else 5
+        a.steps = {"gemv": 2000, "encode": 5, "importance": 20}[a.path]
     if a.warmup is None:
         a.warmup = 10 if a.path == "gemv" else 3
     return a
@@ -649,8 +651,180 @@ def encode_arm(args):
         print(json.dumps(line), flush=True)
 
 
+# ------------------------------------------------------- importance path
+
+IMP_METRIC = "data-free importance + outlier statistics of an FP16 checkpoint: GB/s of weights"
+
+
+def importance_launches(spec) -> int:
+    """Kernels one seedq_importance call launches (gains, head pass and its
+    finishing step, six or seven per layer, rho normalization, ratios)."""
+    per_layer = 6 + (1 if spec.n_heads > spec.n_kv_heads else 0)
+    return (2 * spec.n_layers + 1) + 2 + spec.n_layers * per_layer + 2
+
+
+def importance_oracle_sample(spec, nthreads):
+    """The oracle's work for one layer of the checkpoint (Eq. gamma / prop row
+    sums, the backward proxy's column sums, the outlier statistics of its seven
+    matrices), timed, and scaled to the whole model by weight count.  Returns
+    (seconds for the whole model, description)."""
+    import numpy as np
+
+    sys.path.insert(0, os.path.join(ROOT, "oracle"))
+    import importance as I
+
+    from paper_2609_38477_gb300 import workloads as W
+
+    l = spec.n_layers - 1
+    mats = {k: W.synth_weight_rows(spec, l, k, 0, spec.shape(k)[0]) for k in W.MODEL_KINDS}
+    a_attn = I.a_from_gain(W.synth_gain(spec, l, "attn"))
+    a_mlp = I.a_from_gain(W.synth_gain(spec, l, "mlp"))
+    G = np.ones(spec.d_model)
+    t0 = time.perf_counter()
+    I.a_o(mats["v"], a_attn, spec.n_heads, spec.n_kv_heads)
+    I.a_down(mats["gate"], mats["up"], a_mlp)
+    Gh = I.sq_cols(mats["down"], G)
+    I.sq_cols(mats["gate"], Gh)
+    I.sq_cols(mats["up"], Gh)
+    Ga = I.sq_cols(mats["o"], G)
+    n_rep = spec.n_heads // spec.n_kv_heads
+    I.sq_cols(mats["v"], Ga.reshape(spec.n_kv_heads, n_rep, spec.head_dim).sum(axis=1).ravel())
+    for k in W.MODEL_KINDS:
+        I.dynamic_range(mats[k])
+    dt = time.perf_counter() - t0
+    layer_w = sum(m.size for m in mats.values())
+    desc = (f"oracle (numpy fp64, {nthreads} host threads available) on layer {l} of the "
+            f"checkpoint ({layer_w / 1e6:.0f} M of {spec.weights / 1e6:.0f} M weights: row and "
+            f"column sums of squares, full-sort column medians), scaled by weight count")
+    return dt * spec.weights / layer_w, desc
+
+
+def importance_reference(args):
+    if int(os.environ.get("RANK", "0")) != 0:
+        return
+    from paper_2609_38477_gb300 import workloads as W
+
+    spec = W.MODELS[args.model]
+    cores = cpu_cores()
+    times, desc = [], ""
+    for _ in range(max(1, min(args.steps, 2))):  # each sample is ~10-20 s of host work
+        t, desc = importance_oracle_sample(spec, cores)
+        times.append(t)
+    value = spec.weights * 2 / statistics.mean(times) / 1e9
+    print(json.dumps({
+        "impl": "reference", "metric": IMP_METRIC, "value": value, "unit": "GB/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": 0,
+        "ms_per_step": statistics.mean(times) * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": spec.description},
+        "cpu_baseline": {"value": value, "unit": "GB/s", "cores": cores, "kind": "oracle",
+                         "sample": desc},
+        "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+def importance_arm(args):
+    import torch
+
+    rank, world, local = dist_init()
+    torch.cuda.set_device(local)
+    import __graft_entry__ as GE
+
+    GE.build()
+    from paper_2609_38477_gb300 import workload_gpu as G
+    from paper_2609_38477_gb300 import workloads as W
+
+    spec = W.MODELS[args.model]
+    gm = G.synth_model_device(spec)
+    out = G.importance_buffers(spec, with_stats=False)
+    stream = torch.cuda.current_stream()
+    wbytes = spec.weights * 2
+
+    def step():
+        return G.run_importance(gm, out, 4, stream)
+
+    for _ in range(max(args.warmup, 3)):
+        outliers = step()
+    torch.cuda.synchronize()
+    clocks = Clocks(gpu_index(local))
+    dist_barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    # The checkpoint (13.5 GB for the Llama-2-7B shape) is far larger than L2,
+    # so no flush is needed between passes.  Each pass ends with a host sync
+    # (the outlier selection reads the candidates on the host).
+    for a, b in ev:
+        a.record(stream)
+        step()
+        b.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    dist_barrier()
+    step_ms = dist_max(statistics.mean(a.elapsed_time(b) for a, b in ev))
+
+    # End to end: every weight and gain copied in from pinned host memory, the
+    # tables copied out.
+    dev = [t for y in gm.layers for t in y.values()] + [gm.final_norm, gm.lm_head]
+    host = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in dev]
+    for h, t in zip(host, dev):
+        h.copy_(t)
+    outs = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True) for k, v in out.items()}
+    e2e = []
+    for _ in range(max(1, min(args.steps, 3))):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for h, t in zip(host, dev):
+            t.copy_(h, non_blocking=True)
+        step()
+        for k, v in out.items():
+            outs[k].copy_(v, non_blocking=True)
+        b.record(stream)
+        b.synchronize()
+        e2e.append(a.elapsed_time(b))
+    e2e_ms = dist_max(statistics.mean(e2e))
+    h2d = sum(t.numel() * t.element_size() for t in dev)
+    d2h = sum(v.numel() * v.element_size() for v in out.values())
+
+    pk = measured_peaks()
+    peak = pk["hbm_gbs"] if pk else 6800.0
+    achieved = wbytes / (step_ms * 1e-3) / 1e9
+    line = {
+        "metric": IMP_METRIC, "value": world * achieved, "unit": "GB/s",
+        "n_gpus": world, "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": step_ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "fp32/fp64",
+        "data": "synthetic",
+        "config": {"workload": spec.description, "weights": spec.weights,
+                   "l2": "inputs far larger than L2 (whole checkpoint read once per pass)",
+                   "outliers": [list(o) for o in outliers]},
+        "clocks": clk,
+        "e2e": {"value": world * wbytes / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": args.steps * importance_launches(spec),
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": None,
+                     "kernel": "the whole pass (column passes over every matrix plus the "
+                               "finishing kernels), algorithmic bytes = the FP16 weights once",
+                     "peak_basis": "MEASURED_PEAKS.json hbm_gbs (measured)" if pk else
+                                   "fallback 6800 GB/s"},
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        t, desc = importance_oracle_sample(spec, cpu_cores())
+        line["cpu_baseline"] = {"value": wbytes / t / 1e9, "unit": "GB/s", "cores": cpu_cores(),
+                                "kind": "oracle", "sample": desc}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
+    if args.path == "importance":
+        if args.impl == "reference":
+            importance_reference(args)
+        else:
+            importance_arm(args)
+        return
     if args.path == "encode":
         if args.impl == "reference":
             encode_reference(args)

@@ -597,9 +597,9 @@ struct FinArgs {
   int32_t n_out, n_rep, head_dim;
 };
 
-// Blocks [0, nb_g) update the stream scale; the rest take one output channel
-// of a_down / a_o per warp (tile sums and quadrature split over the lanes,
-// combined by a fixed xor tree).  In E[silu(g)^2] the logistic factor
+// Blocks [0, nb_g) update the stream scale; the rest take 32 output channels
+// of a_down / a_o each (tile sums and quadrature split over 8 thread groups,
+// combined in a fixed order).  In E[silu(g)^2] the logistic factor
 // 1 / (1 + e^-g) is evaluated in float32 (relative error ~1e-7, below the
 // tables' float32 rounding); the node, the product and the sums are fp64.
 __global__ void k_fin(const __grid_constant__ FinArgs f, int nb_g) {
@@ -623,37 +623,64 @@ __global__ void k_fin(const __grid_constant__ FinArgs f, int nb_g) {
     return;
   }
   if (!f.a_out) return;
-  const int lane = threadIdx.x & 31;
-  const int i = ((int)blockIdx.x - nb_g) * (int)(blockDim.x >> 5) + (int)(threadIdx.x >> 5);
-  if (i >= f.n_out) return;
-  if (f.mode == 0) {
-    double v = 0.0, u = 0.0;
-    for (int t = lane; t < f.ntile; t += 32) {
-      v += (double)f.rp0[(int64_t)t * f.nrows + i];
-      u += (double)f.rp1[(int64_t)t * f.nrows + i];
-    }
-    for (int o = 16; o > 0; o >>= 1) {
-      v += __shfl_xor_sync(0xffffffffu, v, o);
-      u += __shfl_xor_sync(0xffffffffu, u, o);
-    }
-    // E[silu(g)^2] with the 64 nodes split over the lanes.
-    const double sd = sqrt(2.0 * v);
-    double acc = 0.0;
-    for (int k = lane; k < kGH; k += 32) {
-      const double g = sd * c_gh_x[k];
-      const float sig = 1.f / (1.f + expf((float)-g));
-      const double y = g * (double)sig;
-      acc = fma(c_gh_w[k], y * y, acc);
-    }
-    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    if (lane == 0) f.a_out[i] = (float)(acc * u);
-  } else {
+  // 32 channels per block: thread (cl, tg) sums the tiles tg, tg + 8, ... of
+  // channel cl (coalesced across cl), the 8 partial sums are added in tg order.
+  __shared__ double red_v[8][32], red_u[8][32];
+  __shared__ double s_sd[32];
+  const int cl = threadIdx.x & 31, tg = threadIdx.x >> 5;
+  const int i = ((int)blockIdx.x - nb_g) * 32 + cl;
+  const bool ok = i < f.n_out;
+  int row = i;
+  if (f.mode == 1 && ok) {
     const int h = i / f.head_dim, o = i - h * f.head_dim;
-    const int row = (h / f.n_rep) * f.head_dim + o;
-    double v = 0.0;
-    for (int t = lane; t < f.ntile; t += 32) v += (double)f.rp0[(int64_t)t * f.nrows + row];
-    for (int k = 16; k > 0; k >>= 1) v += __shfl_xor_sync(0xffffffffu, v, k);
-    if (lane == 0) f.a_out[i] = (float)v;
+    row = (h / f.n_rep) * f.head_dim + o;
+  }
+  double v = 0.0, u = 0.0;
+  if (ok) {
+    for (int t = tg; t < f.ntile; t += 8) {
+      v += (double)f.rp0[(int64_t)t * f.nrows + row];
+      if (f.mode == 0) u += (double)f.rp1[(int64_t)t * f.nrows + row];
+    }
+  }
+  red_v[tg][cl] = v;
+  red_u[tg][cl] = u;
+  __syncthreads();
+  if (tg == 0) {
+    double sv = 0.0, su = 0.0;
+    for (int k = 0; k < 8; ++k) {
+      sv += red_v[k][cl];
+      su += red_u[k][cl];
+    }
+    red_v[0][cl] = sv;
+    red_u[0][cl] = su;
+    if (f.mode == 0) {
+      // sqrt(2 v): float estimate and one fp64 Newton step.
+      const double x = 2.0 * sv;
+      const double r = (double)sqrtf((float)x);
+      s_sd[cl] = r > 0.0 ? 0.5 * (r + x / r) : 0.0;
+    }
+  }
+  __syncthreads();
+  if (f.mode == 1) {
+    if (tg == 0 && ok) f.a_out[i] = (float)red_v[0][cl];
+    return;
+  }
+  // E[silu(g)^2]: the 64 nodes split over the 8 thread groups.
+  const double sd = s_sd[cl];
+  double acc = 0.0;
+  for (int k = tg; k < kGH; k += 8) {
+    const double g = sd * c_gh_x[k];
+    const float sig = 1.f / (1.f + expf((float)-g));
+    const double y = g * (double)sig;
+    acc = fma(c_gh_w[k], y * y, acc);
+  }
+  __syncthreads();
+  red_v[tg][cl] = acc;
+  __syncthreads();
+  if (tg == 0 && ok) {
+    double e = 0.0;
+    for (int k = 0; k < 8; ++k) e += red_v[k][cl];
+    f.a_out[i] = (float)(e * red_u[0][cl]);
   }
 }
 
@@ -1166,7 +1193,7 @@ seedq_status seedq_importance(const seedq_llama_model *m, const seedq_importance
       F.rho_raw = rraw + (size_t)(2 * l) * d; F.d = d;
       F.rp0 = rpa; F.rp1 = rpb; F.ntile = d / kTC; F.nrows = f;
       F.a_out = out->a_down + (size_t)l * f; F.mode = 0; F.n_out = f;
-      k_fin<<<gb + (f + 7) / 8, 256, 0, st>>>(F, gb);
+      k_fin<<<gb + (f + 31) / 32, 256, 0, st>>>(F, gb);
       SEEDQ_CUDA(cudaGetLastError());
       ++step;
     }
@@ -1206,7 +1233,7 @@ seedq_status seedq_importance(const seedq_llama_model *m, const seedq_importance
       F.rp0 = rpa; F.ntile = d / kTC; F.nrows = kvd;
       F.a_out = out->a_o + (size_t)l * qd; F.mode = 1; F.n_out = qd;
       F.n_rep = n_rep; F.head_dim = hd;
-      k_fin<<<gb + (qd + 7) / 8, 256, 0, st>>>(F, gb);
+      k_fin<<<gb + (qd + 31) / 32, 256, 0, st>>>(F, gb);
       SEEDQ_CUDA(cudaGetLastError());
       ++step;
     }
