@@ -213,9 +213,12 @@ def traffic_per_launch(kernel_hash: str):
         return None
 
 
+KERNEL_SOURCES = ("gemv.cu", "seedq_internal.cuh", "cp_async.cuh", "f32x2.cuh")
+
+
 def kernel_source_hash() -> str:
     h = hashlib.sha256()
-    for f in ("gemv.cu", "seedq_internal.cuh"):
+    for f in KERNEL_SOURCES:
         h.update(open(os.path.join(ROOT, "paper_2609_38477_gb300", "csrc", f), "rb").read())
     return h.hexdigest()[:16]
 

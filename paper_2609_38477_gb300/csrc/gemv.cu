@@ -27,6 +27,8 @@
 #include <new>
 #include <vector>
 
+#include "cp_async.cuh"
+#include "f32x2.cuh"
 #include "seedq_internal.cuh"
 
 namespace seedq {
@@ -86,14 +88,6 @@ __host__ __device__ inline int batch_template(int n) {
 
 __device__ __forceinline__ float bf16_to_f32(uint16_t b) { return __uint_as_float((uint32_t)b << 16); }
 
-__device__ __forceinline__ void cp_async16(void *smem_dst, const void *gsrc) {
-  const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d), "l"(gsrc) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
-
 // CTA whose range holds unit u (cb: the ctas + 1 range starts).
 __device__ __forceinline__ int cta_of(const int64_t *cb, int ctas, int64_t u) {
   int lo = 0, hi = ctas - 1;
@@ -103,28 +97,6 @@ __device__ __forceinline__ int cta_of(const int64_t *cb, int ctas, int64_t u) {
     else hi = mid - 1;
   }
   return lo;
-}
-
-// Packed pair of fp32 values (lane-wise fma.rn.f32x2 on sm_100 and later).
-__device__ __forceinline__ uint64_t pk2(float a, float b) {
-  uint64_t r;
-  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
-  return r;
-}
-__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
-  uint64_t d;
-  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
-  return d;
-}
-__device__ __forceinline__ uint64_t mul2(uint64_t a, uint64_t b) {
-  uint64_t d;
-  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-  return d;
-}
-__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b) {
-  uint64_t d;
-  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-  return d;
 }
 
 // One block: reconstruct its 8 weights and add scale * sum_i I_i x_b[i] to
@@ -153,18 +125,18 @@ __device__ __forceinline__ void block_fma(const uint32_t (&w)[3], uint32_t sh, c
     const uint64_t *x2 = reinterpret_cast<const uint64_t *>(xc);  // pairs of batch columns
     uint64_t Ip[8];
 #pragma unroll
-    for (int i = 0; i < 8; ++i) Ip[i] = pk2(I[i], I[i]);
-    const uint64_t sp = pk2(scale, scale);
+    for (int i = 0; i < 8; ++i) Ip[i] = f2_pack(I[i], I[i]);
+    const uint64_t sp = f2_pack(scale, scale);
 #pragma unroll
     for (int q = 0; q < NB / 2; ++q) {
-      uint64_t s0 = mul2(Ip[0], x2[0 * (NB / 2) + q]), s1 = mul2(Ip[4], x2[4 * (NB / 2) + q]);
-      s0 = fma2(Ip[1], x2[1 * (NB / 2) + q], s0);
-      s1 = fma2(Ip[5], x2[5 * (NB / 2) + q], s1);
-      s0 = fma2(Ip[2], x2[2 * (NB / 2) + q], s0);
-      s1 = fma2(Ip[6], x2[6 * (NB / 2) + q], s1);
-      s0 = fma2(Ip[3], x2[3 * (NB / 2) + q], s0);
-      s1 = fma2(Ip[7], x2[7 * (NB / 2) + q], s1);
-      const uint64_t a = fma2(sp, add2(s0, s1), pk2(acc[2 * q], acc[2 * q + 1]));
+      uint64_t s0 = f2_mul(Ip[0], x2[0 * (NB / 2) + q]), s1 = f2_mul(Ip[4], x2[4 * (NB / 2) + q]);
+      s0 = f2_fma(Ip[1], x2[1 * (NB / 2) + q], s0);
+      s1 = f2_fma(Ip[5], x2[5 * (NB / 2) + q], s1);
+      s0 = f2_fma(Ip[2], x2[2 * (NB / 2) + q], s0);
+      s1 = f2_fma(Ip[6], x2[6 * (NB / 2) + q], s1);
+      s0 = f2_fma(Ip[3], x2[3 * (NB / 2) + q], s0);
+      s1 = f2_fma(Ip[7], x2[7 * (NB / 2) + q], s1);
+      const uint64_t a = f2_fma(sp, f2_add(s0, s1), f2_pack(acc[2 * q], acc[2 * q + 1]));
       acc[2 * q] = __uint_as_float((uint32_t)a);
       acc[2 * q + 1] = __uint_as_float((uint32_t)(a >> 32));
     }

@@ -25,7 +25,7 @@
 // fp32-rounded weight is rounded once, 16 rows accumulate in fp32 and then in
 // fp64 (relative error of a column sum below 18 u, u = 2^-24, all terms being
 // non-negative), partial row sums of 32 columns are fp32 and their tile sums
-// fp64; the stream scale stays fp64.  Tables are rounded to float32 (App.
+// compensated float32 sums; the stream scale stays fp64.  Tables are rounded to float32 (App.
 // A.7).  The outlier statistics are exact: maxima and medians are FP16 values,
 // the statistic is one IEEE division of their fp64 sum, and the activation
 // mean is the correctly rounded sum divided by the count.
@@ -38,6 +38,7 @@
 #include <algorithm>
 #include <vector>
 
+#include "cp_async.cuh"
 #include "f32x2.cuh"
 #include "seedq_internal.cuh"
 #include "synth.cuh"
@@ -59,8 +60,21 @@ constexpr double kEpsDR = 5.9604644775390625e-08;  // 2^-24
 constexpr double kDrMin = 1.0e3;
 constexpr double kActMin = 1.0e2;
 
-__constant__ double c_gh_x[kGH];  // nodes
-__constant__ double c_gh_w[kGH];  // weights / sqrt(pi)
+__constant__ float c_gh_xf[kGH];  // Gauss-Hermite nodes
+__constant__ float c_gh_wf[kGH];  // weights / sqrt(pi)
+
+// Compensated float32 sum (Kahan): s + (-c) carries the running sum to a few
+// units in the last place independently of the number of terms.
+struct Kahan {
+  float s = 0.f, c = 0.f;
+  __device__ __forceinline__ void add(float x) {
+    const float y = __fsub_rn(x, c);
+    const float t = __fadd_rn(s, y);
+    c = __fsub_rn(__fsub_rn(t, s), y);
+    s = t;
+  }
+  __device__ __forceinline__ double value() const { return (double)s - (double)c; }
+};
 
 struct Cand {
   double v;
@@ -106,18 +120,6 @@ __device__ __forceinline__ uint4 ld_stream16(const void *p) {
                : "l"(p));
   return v;
 }
-
-__device__ __forceinline__ void cp_async16(void *smem_dst, const void *gsrc) {
-  const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d), "l"(gsrc) : "memory");
-}
-__device__ __forceinline__ void cp_async4(void *smem_dst, const void *gsrc) {
-  const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
-  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(d), "l"(gsrc) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
 
 __device__ __forceinline__ uint4 lds128(const uint4 *p) {
   uint4 v;
@@ -599,9 +601,9 @@ struct FinArgs {
 
 // Blocks [0, nb_g) update the stream scale; the rest take 32 output channels
 // of a_down / a_o each (tile sums and quadrature split over 8 thread groups,
-// combined in a fixed order).  In E[silu(g)^2] the logistic factor
-// 1 / (1 + e^-g) is evaluated in float32 (relative error ~1e-7, below the
-// tables' float32 rounding); the node, the product and the sums are fp64.
+// combined in a fixed order).  E[silu(g)^2] is evaluated in float32 (each
+// term to a few units in the last place, the sum compensated), below the
+// tables' tolerance.
 __global__ void k_fin(const __grid_constant__ FinArgs f, int nb_g) {
   if ((int)blockIdx.x < nb_g) {
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
@@ -624,9 +626,12 @@ __global__ void k_fin(const __grid_constant__ FinArgs f, int nb_g) {
   }
   if (!f.a_out) return;
   // 32 channels per block: thread (cl, tg) sums the tiles tg, tg + 8, ... of
-  // channel cl (coalesced across cl), the 8 partial sums are added in tg order.
-  __shared__ double red_v[8][32], red_u[8][32];
-  __shared__ double s_sd[32];
+  // channel cl (coalesced across cl); the 8 partial sums are combined in tg
+  // order.  All sums are compensated float32 sums (Kahan), accurate to a few
+  // units in the last place whatever their length, on the wide float32 pipe.
+  __shared__ float red_v[8][32], red_vc[8][32], red_u[8][32], red_uc[8][32];
+  __shared__ float s_sd[32];
+  __shared__ double s_u[32];
   const int cl = threadIdx.x & 31, tg = threadIdx.x >> 5;
   const int i = ((int)blockIdx.x - nb_g) * 32 + cl;
   const bool ok = i < f.n_out;
@@ -635,52 +640,53 @@ __global__ void k_fin(const __grid_constant__ FinArgs f, int nb_g) {
     const int h = i / f.head_dim, o = i - h * f.head_dim;
     row = (h / f.n_rep) * f.head_dim + o;
   }
-  double v = 0.0, u = 0.0;
+  Kahan v, u;
   if (ok) {
     for (int t = tg; t < f.ntile; t += 8) {
-      v += (double)f.rp0[(int64_t)t * f.nrows + row];
-      if (f.mode == 0) u += (double)f.rp1[(int64_t)t * f.nrows + row];
+      v.add(f.rp0[(int64_t)t * f.nrows + row]);
+      if (f.mode == 0) u.add(f.rp1[(int64_t)t * f.nrows + row]);
     }
   }
-  red_v[tg][cl] = v;
-  red_u[tg][cl] = u;
+  red_v[tg][cl] = v.s; red_vc[tg][cl] = v.c;
+  red_u[tg][cl] = u.s; red_uc[tg][cl] = u.c;
   __syncthreads();
   if (tg == 0) {
-    double sv = 0.0, su = 0.0;
+    Kahan sv, su;
     for (int k = 0; k < 8; ++k) {
-      sv += red_v[k][cl];
-      su += red_u[k][cl];
+      sv.add(red_v[k][cl]);
+      sv.add(-red_vc[k][cl]);
+      su.add(red_u[k][cl]);
+      su.add(-red_uc[k][cl]);
     }
-    red_v[0][cl] = sv;
-    red_u[0][cl] = su;
-    if (f.mode == 0) {
-      // sqrt(2 v): float estimate and one fp64 Newton step.
-      const double x = 2.0 * sv;
-      const double r = (double)sqrtf((float)x);
-      s_sd[cl] = r > 0.0 ? 0.5 * (r + x / r) : 0.0;
+    const double vv = sv.value(), uu = su.value();
+    if (f.mode == 1) {
+      if (ok) f.a_out[i] = (float)vv;
+    } else {
+      s_sd[cl] = sqrtf((float)(2.0 * vv));
+      s_u[cl] = uu;
     }
   }
+  if (f.mode == 1) return;
   __syncthreads();
-  if (f.mode == 1) {
-    if (tg == 0 && ok) f.a_out[i] = (float)red_v[0][cl];
-    return;
-  }
-  // E[silu(g)^2]: the 64 nodes split over the 8 thread groups.
-  const double sd = s_sd[cl];
-  double acc = 0.0;
+  // E[silu(g)^2]: the 64 nodes split over the 8 thread groups, float32.
+  const float sd = s_sd[cl];
+  Kahan acc;
   for (int k = tg; k < kGH; k += 8) {
-    const double g = sd * c_gh_x[k];
-    const float sig = 1.f / (1.f + expf((float)-g));
-    const double y = g * (double)sig;
-    acc = fma(c_gh_w[k], y * y, acc);
+    const float g = sd * c_gh_xf[k];
+    const float y = g / (1.f + expf(-g));
+    acc.add(c_gh_wf[k] * (y * y));
   }
   __syncthreads();
-  red_v[tg][cl] = acc;
+  red_v[tg][cl] = acc.s;
+  red_vc[tg][cl] = acc.c;
   __syncthreads();
   if (tg == 0 && ok) {
-    double e = 0.0;
-    for (int k = 0; k < 8; ++k) e += red_v[k][cl];
-    f.a_out[i] = (float)(e * red_u[0][cl]);
+    Kahan e;
+    for (int k = 0; k < 8; ++k) {
+      e.add(red_v[k][cl]);
+      e.add(-red_vc[k][cl]);
+    }
+    f.a_out[i] = (float)(e.value() * s_u[cl]);
   }
 }
 
@@ -983,10 +989,19 @@ struct DevBuf {
   }
 };
 
-// The 64-node rule, computed once per process.
-const double *gh_rule() {
-  static double table[2 * kGH];
-  static const bool done = (gauss_hermite(kGH, table, table + kGH), true);
+// The 64-node rule (nodes, then weights / sqrt(pi)) in float32, computed once
+// per process in fp64.
+const float *gh_rule() {
+  static float table[2 * kGH];
+  static const bool done = [] {
+    double x[kGH], w[kGH];
+    gauss_hermite(kGH, x, w);
+    for (int k = 0; k < kGH; ++k) {
+      table[k] = (float)x[k];
+      table[kGH + k] = (float)w[k];
+    }
+    return true;
+  }();
   (void)done;
   return table;
 }
@@ -1114,9 +1129,9 @@ seedq_status seedq_importance(const seedq_llama_model *m, const seedq_importance
   if (rc != SEEDQ_OK) return rc;
   Cand *cand_dr = cand, *cand_act = cand + total_cols;
   SEEDQ_CUDA(cudaMemsetAsync(S.arrive, 0, sizeof(uint32_t) * S.arrive_cap, st));
-  SEEDQ_CUDA(cudaMemcpyToSymbolAsync(c_gh_x, gh_rule(), sizeof(double) * kGH, 0,
+  SEEDQ_CUDA(cudaMemcpyToSymbolAsync(c_gh_xf, gh_rule(), sizeof(float) * kGH, 0,
                                      cudaMemcpyHostToDevice, st));
-  SEEDQ_CUDA(cudaMemcpyToSymbolAsync(c_gh_w, gh_rule() + kGH, sizeof(double) * kGH, 0,
+  SEEDQ_CUDA(cudaMemcpyToSymbolAsync(c_gh_wf, gh_rule() + kGH, sizeof(float) * kGH, 0,
                                      cudaMemcpyHostToDevice, st));
   SEEDQ_CUDA(cudaMemsetAsync(ncand, 0, 2 * sizeof(uint32_t), st));
   SEEDQ_CUDA(cudaMemsetAsync(gexp, 0x80, sizeof(int) * (2 * L + 1), st));  // below any exponent
