@@ -84,7 +84,7 @@ struct Cand {
 // Partial results of one (slab, tile) work item of the column pass.
 struct Part {
   double cs[kTC];
-  uint32_t mx[kTC], m0[kTC], cnt[kTC];  // cnt: elements >= the slab's threshold
+  uint32_t mx[kTC], m0[kTC], cnt[kTC];  // cnt: elements below the slab's threshold
 };
 
 struct ColJob {
@@ -139,7 +139,7 @@ __device__ __forceinline__ double half_val(uint32_t bits) {
 // 1e3 (K = 16), and counts |W| < U0_s while it streams.  With M0 = min_s M0_s
 // (whose threshold U0 is the smallest), if the column maximum M <= K M0 and
 // the counts sum to at most (R-1)/2, then at most (R-1)/2 elements lie below
-// U0, both middle order statistics are >= U0, and max / (median + eps) <=
+// U0 (the counts are FP16 compares of FP16 magnitudes, exact), both middle order statistics are >= U0, and max / (median + eps) <=
 // 1e3 / 2.01: the column cannot qualify.  Every other column gets its exact
 // median.
 constexpr float kGrowth = 16.f;
@@ -150,8 +150,8 @@ struct Acc {
   uint64_t cf[4];   // current fp32 chunk, packed pairs
   uint64_t av[4];   // row-sum weights a_c, packed pairs
   uint32_t mx[4];   // packed maxima of |W| bits
-  uint32_t cnt[4];  // packed counts of |W| >= U0
-  uint32_t u0[4];   // packed thresholds
+  __half2 cnt[4];   // counts of |W| < U0 (small integers, exact in FP16)
+  __half2 u0[4];    // thresholds
 };
 
 // The thread's rows of one stage (kFull: all 8 valid, else the first nu);
@@ -172,10 +172,10 @@ __device__ __forceinline__ void stage_rows(const uint4 *slot, const float *wst, 
     uint64_t rs = 0;
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-      A.mx[q] = __vmaxu2(A.mx[q], wd[q] & 0x7fff7fffu);
-      // Per 16-bit lane 0x8000 + |w| - U0 (no borrow across lanes): bit 15
-      // set iff |w| >= U0.
-      A.cnt[q] += ((((wd[q] | 0x80008000u) - A.u0[q]) >> 15) & 0x00010001u);
+      const uint32_t m = wd[q] & 0x7fff7fffu;  // |w| as FP16 bits
+      A.mx[q] = __vmaxu2(A.mx[q], m);
+      // Count |w| < U0 in FP16 (exact integers up to 2048 per thread and item).
+      A.cnt[q] = __hadd2(A.cnt[q], __hlt2(*reinterpret_cast<const __half2 *>(&m), A.u0[q]));
       if (kCols || kRows) {
         const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&wd[q]));
         const uint64_t f2 = f2_pack(f.x, f.y);
@@ -484,8 +484,10 @@ __global__ void __launch_bounds__(kCT, 2) k_colpass(const __grid_constant__ ColA
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         acc.cf[q] = 0;
-        acc.mx[q] = acc.cnt[q] = 0u;
-        acc.u0[q] = s_u0[lc0 + 2 * q] | (s_u0[lc0 + 2 * q + 1] << 16);
+        acc.mx[q] = 0u;
+        acc.cnt[q] = __float2half2_rn(0.f);
+        const uint32_t u2 = s_u0[lc0 + 2 * q] | (s_u0[lc0 + 2 * q + 1] << 16);
+        acc.u0[q] = *reinterpret_cast<const __half2 *>(&u2);
         acc.av[q] = rows ? f2_pack(J.a[ci.tile * kTC + lc0 + 2 * q], J.a[ci.tile * kTC + lc0 + 2 * q + 1])
                          : 0;
       }
@@ -519,7 +521,13 @@ __global__ void __launch_bounds__(kCT, 2) k_colpass(const __grid_constant__ ColA
         __syncthreads();
       }
       cta_reduce16<true>(acc.mx, buf, s_max);
-      cta_reduce16<false>(acc.cnt, buf, s_cnt);
+      uint32_t cnt[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float2 c = __half22float2(acc.cnt[q]);
+        cnt[q] = (uint32_t)c.x | ((uint32_t)c.y << 16);
+      }
+      cta_reduce16<false>(cnt, buf, s_cnt);
       if (t < kTC) {
         P.mx[t] = s_max[t];
         P.m0[t] = s_m0[t];
@@ -539,14 +547,13 @@ __global__ void __launch_bounds__(kCT, 2) k_colpass(const __grid_constant__ ColA
           const int64_t col = (int64_t)ci.tile * kTC + t;
           const Part *ps = J.part + (int64_t)ci.tile * J.slabs;
           double sum = 0.0;
-          uint32_t m = 0, mn = 0xffffu, ge = 0;
+          uint32_t m = 0, mn = 0xffffu, n = 0;  // n: elements below their slab's threshold
           for (int s2 = 0; s2 < J.slabs; ++s2) {
             if (cols) sum += __ldcg(&ps[s2].cs[t]);
             m = max(m, __ldcg(&ps[s2].mx[t]));
             mn = min(mn, __ldcg(&ps[s2].m0[t]));
-            ge += __ldcg(&ps[s2].cnt[t]);
+            n += __ldcg(&ps[s2].cnt[t]);
           }
-          const uint32_t n = (uint32_t)J.R - ge;  // elements below their slab's threshold
           if (cols) {
             J.colsum[col] = sum;
             if (J.colsum_f) J.colsum_f[col] = (float)sum;
@@ -903,7 +910,8 @@ bool aligned16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
 int64_t slab_rows_for(int64_t row_tiles, int ctas) {
   int64_t h = row_tiles / ((int64_t)kItemsPerCta * ctas);
   h = (h + kStageRows - 1) / kStageRows * kStageRows;
-  return h < kStageRows ? kStageRows : h;
+  // At most 2048 rows per thread and item, so the FP16 counts stay exact.
+  return h < kStageRows ? kStageRows : std::min<int64_t>(h, 2048 * kPhases);
 }
 int64_t items_of(int64_t R, int64_t C, int64_t h) { return (C / kTC) * ((R + h - 1) / h); }
 
