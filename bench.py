@@ -38,7 +38,7 @@ def parse():
     p.add_argument("--workload", default="c1")
     p.add_argument("--batch", type=int, default=1)
     p.add_argument("--no-cpu-baseline", action="store_true")
-    p.add_argument("--path", choices=["gemv", "encode", "importance"], default="gemv",
+    p.add_argument("--path", choices=["gemv", "encode", "importance", "allocate"], default="gemv",
                    help="gemv: the fused decode + GEMV step (default); encode: the exhaustive "
                         "seed-search encoder")
     p.add_argument("--rung", default="16,3", help="encoder rung S,k")
@@ -47,7 +47,7 @@ def parse():
                    help="synthetic FP16 checkpoint of the importance path")
     a = p.parse_args()
     if a.steps is None:
-        a.steps = {"gemv": 2000, "encode": 5, "importance": 20}[a.path]
+        a.steps = {"gemv": 2000, "encode": 5, "importance": 20, "allocate": 5}[a.path]
     if a.warmup is None:
         a.warmup = 10 if a.path == "gemv" else 3
     return a
@@ -820,8 +820,136 @@ def importance_arm(args):
         print(json.dumps(line), flush=True)
 
 
+# --------------------------------------------------------- allocator path
+
+ALLOC_METRIC = "Alg. 1 allocation over a model's tensors (floor, multiplier bisection, tie pass)"
+
+
+def allocate_inputs(name):
+    from paper_2609_38477_gb300 import workloads as W
+
+    w = W.WORKLOADS[name]
+    d = load_schedule(name)
+    factors = []
+    for i, t in enumerate(w.tensors):
+        a, rho = W.importance(w, i)
+        factors.append((t.R, t.C, a, rho))
+    return w, d, factors
+
+
+def allocate_oracle(name, w, d):
+    sys.path.insert(0, os.path.join(ROOT, "oracle"))
+    import oracle as O
+    from paper_2609_38477_gb300 import workloads as W
+
+    ts = [O.Tensor(t.R, t.C, *W.importance(w, i)) for i, t in enumerate(w.tensors)]
+    t0 = time.perf_counter()
+    O.allocate(ts, [tuple(r) for r in d["rungs"]], d["slopes"], d["rbar"], d["floor_f"])
+    return time.perf_counter() - t0
+
+
+def allocate_reference(args):
+    if int(os.environ.get("RANK", "0")) != 0:
+        return
+    w, d, _ = allocate_inputs(args.workload)
+    times = [allocate_oracle(args.workload, w, d) for _ in range(max(1, min(args.steps, 3)))]
+    value = 1.0 / statistics.mean(times)
+    print(json.dumps({
+        "impl": "reference", "metric": ALLOC_METRIC, "value": value, "unit": "allocations/s",
+        "n_gpus": args.gpus, "steps": len(times), "warmup": 0,
+        "ms_per_step": statistics.mean(times) * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": f"{w.name}: {w.description}", "tensors": len(w.tensors)},
+        "cpu_baseline": {"value": value, "unit": "allocations/s", "cores": 1, "kind": "oracle",
+                         "sample": "the oracle's allocator (C, one thread) on the whole tensor set"},
+        "e2e": {"value": value, "unit": "allocations/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+def allocate_arm(args):
+    import torch
+
+    rank, world, local = dist_init()
+    torch.cuda.set_device(local)
+    import __graft_entry__ as GE
+
+    GE.build()
+    from paper_2609_38477_gb300 import seedq as Q
+
+    w, d, factors = allocate_inputs(args.workload)
+    rungs = [tuple(r) for r in d["rungs"]]
+
+    def step():
+        return Q.allocate(factors, rungs, d["slopes"], d["rbar"], d["floor_f"])
+
+    for _ in range(max(args.warmup, 3)):
+        got = step()
+    assert list(got[0]) == d["theta"] and [int(x) for x in got[3]] == d["tie_count"]
+    # Latency floor of one bisection step: a launch, an 8-byte read-back and a
+    # host synchronization (the allocator needs the count before the next step).
+    one = torch.zeros(1, dtype=torch.int16, device="cuda")
+    host = torch.zeros(1, dtype=torch.int16, pin_memory=True)
+    for _ in range(20):
+        Q.synth_fp16(0, 0, 1, 1, 0, one)
+        host.copy_(one, non_blocking=True)
+        torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(200):
+        Q.synth_fp16(0, 0, 1, 1, 0, one)
+        host.copy_(one, non_blocking=True)
+        torch.cuda.synchronize()
+    rt = (time.perf_counter() - t0) / 200
+    clocks = Clocks(gpu_index(local))
+    dist_barrier()
+    clocks.start()
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        step()
+        times.append(time.perf_counter() - t0)
+    clk = clocks.stop()
+    step_s = dist_max(statistics.mean(times))
+    # Evaluations: the floor's and the multiplier's bisections over 64-bit
+    # patterns, plus the two end points, the tied group and the demotion counts.
+    evals = 64 + 64 + 5
+    line = {
+        "metric": ALLOC_METRIC, "value": world / step_s, "unit": "allocations/s",
+        "n_gpus": world, "steps": args.steps, "warmup": max(args.warmup, 3),
+        "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": f"{w.name}: {w.description}", "tensors": len(w.tensors),
+                   "timing": "host wall clock around the synchronous call (it includes the "
+                             "factor upload and kernels and ~130 dependent evaluations)"},
+        "clocks": clk,
+        "e2e": {"value": world / step_s, "unit": "allocations/s",
+                "h2d_bytes_per_step": sum(4 * (C + (R if rho is not None else 0))
+                                          for R, C, a, rho in factors),
+                "d2h_bytes_per_step": 8 * (1 + len(factors) + 9) * evals},
+        "gpu_launches": args.steps * (3 * len(factors) + evals),
+        "roofline": {"bound": "latency", "achieved": evals / step_s, "peak": 1.0 / rt,
+                     "unit": "dependent evaluations/s", "frac": rt * evals / step_s,
+                     "traffic": None, "kernel": "k_alloc_eval (one per bisection step)",
+                     "peak_basis": "measured launch + 8-byte read-back + synchronize round trip "
+                                   f"({rt * 1e6:.1f} us)"},
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        t = allocate_oracle(args.workload, w, d)
+        line["cpu_baseline"] = {"value": 1.0 / t, "unit": "allocations/s", "cores": 1,
+                                "kind": "oracle",
+                                "sample": "the oracle's allocator (C, one thread) on the whole set"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
+    if args.path == "allocate":
+        if args.impl == "reference":
+            allocate_reference(args)
+        else:
+            allocate_arm(args)
+        return
     if args.path == "importance":
         if args.impl == "reference":
             importance_reference(args)

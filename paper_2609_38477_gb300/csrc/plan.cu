@@ -39,10 +39,12 @@ static const uint32_t kTaps[17] = {0, 0, 0, 0, 0, 0, 0, 0,
 // ------------------------------------------------------------ plan kernels
 
 // Stable ascending rank of a: perm[rank(i)] = i with ties broken by index
-// (Sec. 3.3: channels sorted by a before blocking).
-__global__ void k_perm(const float *__restrict__ a, int C, int32_t *__restrict__ perm) {
+// (Sec. 3.3: channels sorted by a before blocking).  blk: this block's index
+// among the ceil(C / blockDim.x) blocks of the tensor.
+__device__ __forceinline__ void perm_block(const float *__restrict__ a, int C, int blk,
+                                           int32_t *__restrict__ perm) {
   __shared__ float tile[1024];
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  const int i = blk * blockDim.x + threadIdx.x;
   const float ai = (i < C) ? a[i] : 0.f;
   int rank = 0;
   for (int base = 0; base < C; base += 1024) {
@@ -57,6 +59,10 @@ __global__ void k_perm(const float *__restrict__ a, int C, int32_t *__restrict__
     }
   }
   if (i < C) perm[rank] = i;
+}
+
+__global__ void k_perm(const float *__restrict__ a, int C, int32_t *__restrict__ perm) {
+  perm_block(a, C, blockIdx.x, perm);
 }
 
 // Row order for the fused kernel: rows with equal or nearby rung breakpoints
@@ -94,8 +100,9 @@ __global__ void k_invperm(const int32_t *__restrict__ perm, int C, int32_t *__re
 
 // Block means of the permuted a, summed in channel order, and their unit-mean
 // normalization summed in ascending block order (Eq. imp; App. A.7 fixed order).
-__global__ void k_abar(const float *__restrict__ a, const int32_t *__restrict__ perm,
-                       int nb, double *__restrict__ abar) {
+// One thread block per tensor.
+__device__ __forceinline__ void abar_block(const float *__restrict__ a, const int32_t *__restrict__ perm,
+                                           int nb, double *__restrict__ abar) {
   __shared__ double mean;
   for (int c = threadIdx.x; c < nb; c += blockDim.x) {
     double s = 0.0;
@@ -112,8 +119,14 @@ __global__ void k_abar(const float *__restrict__ a, const int32_t *__restrict__ 
   for (int c = threadIdx.x; c < nb; c += blockDim.x) abar[c] = __ddiv_rn(abar[c], mean);
 }
 
+__global__ void k_abar(const float *__restrict__ a, const int32_t *__restrict__ perm,
+                       int nb, double *__restrict__ abar) {
+  abar_block(a, perm, nb, abar);
+}
+
 // Row factor normalized to unit mean, summed in ascending row order.
-__global__ void k_rho(const float *__restrict__ rho_in, int64_t R, double *__restrict__ rho) {
+__device__ __forceinline__ void rho_block(const float *__restrict__ rho_in, int64_t R,
+                                          double *__restrict__ rho) {
   __shared__ double mean;
   if (threadIdx.x == 0) {
     double s = 0.0;
@@ -124,6 +137,40 @@ __global__ void k_rho(const float *__restrict__ rho_in, int64_t R, double *__res
   __syncthreads();
   for (int64_t r = threadIdx.x; r < R; r += blockDim.x)
     rho[r] = rho_in ? __ddiv_rn((double)rho_in[r], mean) : 1.0;
+}
+
+__global__ void k_rho(const float *__restrict__ rho_in, int64_t R, double *__restrict__ rho) {
+  rho_block(rho_in, R, rho);
+}
+
+// The same three steps for many tensors at once (the allocator's factors).
+struct FacJob {
+  const float *a;       // C
+  const float *rho_in;  // R, or nullptr
+  int32_t *perm;        // C
+  double *abar;         // C / 8
+  double *rho;          // R
+  int64_t R;
+  int32_t C;
+  int32_t blk0;         // first block of this tensor in k_perm_multi
+};
+
+__global__ void k_perm_multi(const FacJob *__restrict__ jobs, int nt) {
+  int lo = 0, hi = nt - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (jobs[mid].blk0 <= (int)blockIdx.x) lo = mid;
+    else hi = mid - 1;
+  }
+  const FacJob &J = jobs[lo];
+  perm_block(J.a, J.C, blockIdx.x - J.blk0, J.perm);
+}
+
+__global__ void k_factors_multi(const FacJob *__restrict__ jobs) {
+  const FacJob &J = jobs[blockIdx.x];
+  abar_block(J.a, J.perm, J.C / 8, J.abar);
+  __syncthreads();
+  rho_block(J.rho_in, J.R, J.rho);
 }
 
 struct SchedArgs {
@@ -970,7 +1017,8 @@ extern "C" seedq_status seedq_allocate(const seedq_factor_desc *tensors, int32_t
   }
   cudaStream_t st = (cudaStream_t)cuda_stream;
 
-  // Factors of every tensor, exactly as the plan computes them.
+  // Factors of every tensor, exactly as the plan computes them: one device
+  // allocation, one upload of all a and rho, three launches for all tensors.
   std::vector<void *> owned;
   auto cleanup = [&]() {
     for (void *p : owned) cudaFree(p);
@@ -984,37 +1032,65 @@ extern "C" seedq_status seedq_allocate(const seedq_factor_desc *tensors, int32_t
     owned.push_back(p);
     return p;
   };
+  int64_t n_a = 0, n_rho = 0, n_rows = 0, n_nb = 0, blocks = 0;
+  for (int t = 0; t < count; ++t) {
+    n_a += tensors[t].cols;
+    n_rho += tensors[t].rho ? tensors[t].rows : 0;
+    n_rows += tensors[t].rows;
+    n_nb += tensors[t].cols / 8;
+    blocks += (tensors[t].cols + 255) / 256;
+  }
+  std::vector<float> h_in((size_t)(n_a + n_rho));
+  float *d_in = (float *)dalloc(sizeof(float) * (size_t)(n_a + n_rho));
+  int32_t *d_perm = (int32_t *)dalloc(sizeof(int32_t) * (size_t)n_a);
+  double *d_abar = (double *)dalloc(sizeof(double) * (size_t)n_nb);
+  double *d_rho = (double *)dalloc(sizeof(double) * (size_t)n_rows);
+  FacJob *d_jobs = (FacJob *)dalloc(sizeof(FacJob) * count);
+  if (!d_in || !d_perm || !d_abar || !d_rho || !d_jobs) {
+    cleanup();
+    return SEEDQ_ERR_NOMEM;
+  }
+  std::vector<FacJob> hj(count);
   std::vector<AllocTensor> ht(count);
   int64_t rows_total = 0;
-  for (int t = 0; t < count; ++t) {
-    const seedq_factor_desc &d = tensors[t];
-    const int64_t R = d.rows, C = d.cols;
-    const int nb = (int)(C / 8);
-    float *a_in = (float *)dalloc(sizeof(float) * C);
-    float *rho_in = d.rho ? (float *)dalloc(sizeof(float) * R) : nullptr;
-    int32_t *perm = (int32_t *)dalloc(sizeof(int32_t) * C);
-    double *abar = (double *)dalloc(sizeof(double) * nb);
-    double *rho = (double *)dalloc(sizeof(double) * R);
-    if (!a_in || (d.rho && !rho_in) || !perm || !abar || !rho) {
-      cleanup();
-      return SEEDQ_ERR_NOMEM;
+  {
+    int64_t oa = 0, orh = n_a, orow = 0, onb = 0;
+    int32_t b0 = 0;
+    for (int t = 0; t < count; ++t) {
+      const seedq_factor_desc &d = tensors[t];
+      memcpy(h_in.data() + oa, d.a, sizeof(float) * d.cols);
+      const float *rho_dev = nullptr;
+      if (d.rho) {
+        memcpy(h_in.data() + orh, d.rho, sizeof(float) * d.rows);
+        rho_dev = d_in + orh;
+        orh += d.rows;
+      }
+      hj[t] = FacJob{d_in + oa, rho_dev, d_perm + oa, d_abar + onb, d_rho + orow, d.rows,
+                     (int32_t)d.cols, b0};
+      ht[t] = AllocTensor{d_abar + onb, d_rho + orow, d.rows, rows_total, d.rho ? (int32_t)d.rows : 1,
+                          (int32_t)(d.cols / 8)};
+      rows_total += ht[t].nrows;
+      b0 += (int32_t)((d.cols + 255) / 256);
+      oa += d.cols;
+      orow += d.rows;
+      onb += d.cols / 8;
     }
-    cudaError_t e = cudaMemcpyAsync(a_in, d.a, sizeof(float) * C, cudaMemcpyHostToDevice, st);
-    if (e == cudaSuccess && d.rho)
-      e = cudaMemcpyAsync(rho_in, d.rho, sizeof(float) * R, cudaMemcpyHostToDevice, st);
+  }
+  {
+    cudaError_t e = cudaMemcpyAsync(d_in, h_in.data(), sizeof(float) * h_in.size(),
+                                    cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(d_jobs, hj.data(), sizeof(FacJob) * count, cudaMemcpyHostToDevice, st);
     if (e == cudaSuccess) {
-      k_perm<<<(int)((C + 255) / 256), 256, 0, st>>>(a_in, (int)C, perm);
-      k_abar<<<1, 1024, 0, st>>>(a_in, perm, nb, abar);
-      k_rho<<<1, 1024, 0, st>>>(rho_in, R, rho);
+      k_perm_multi<<<(int)blocks, 256, 0, st>>>(d_jobs, count);
+      k_factors_multi<<<count, 1024, 0, st>>>(d_jobs);
       e = cudaGetLastError();
     }
-    if (e == cudaSuccess) e = cudaStreamSynchronize(st);  // host inputs may go out of scope
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);  // h_in is pageable and goes out of scope
     if (e != cudaSuccess) {
       cleanup();
       return cuda_fail(e);
     }
-    ht[t] = AllocTensor{abar, rho, R, rows_total, d.rho ? (int32_t)R : 1, nb};
-    rows_total += ht[t].nrows;
   }
   AllocTensor *dt = (AllocTensor *)dalloc(sizeof(AllocTensor) * count);
   unsigned long long *dev = (unsigned long long *)dalloc(sizeof(unsigned long long) * (1 + count + kMaxJ));
