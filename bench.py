@@ -468,6 +468,13 @@ def our_arm(args):
         el = (time.perf_counter() - t0) / reps
         line["cpu_baseline"] = {"value": n / (el / frac), "unit": "tokens/s", "cores": used,
                                 "kind": "oracle", "sample": desc + f"; {reps} repetitions"}
+        # The same oracle on one host thread (a smaller row sample, ~5 s).
+        run1, frac1, desc1 = oracle_sample(w, sched, n, 5.0, 1)
+        t0 = time.perf_counter()
+        run1()
+        el1 = time.perf_counter() - t0
+        line["cpu_baseline"]["single_thread"] = {"value": n / (el1 / frac1), "unit": "tokens/s",
+                                                 "cores": 1, "sample": desc1}
     if rank == 0:
         print(json.dumps(line), flush=True)
     if lset is not None:
