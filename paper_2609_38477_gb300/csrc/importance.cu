@@ -52,7 +52,7 @@ constexpr int kPhases = kCT / 4;               // row phases (4 threads x 8 colu
 constexpr int kUnroll = 8;                     // rows per thread per stage
 constexpr int kStageRows = kUnroll * kPhases;  // 512
 constexpr int kRing = 3;                       // stages in the ring
-constexpr int kItemsPerCta = 2;                // work items per CTA a launch aims for
+constexpr int kItemsPerCta = 1;                // work items per CTA a launch aims for
 constexpr int kHS = 257;                       // histogram row stride (bank spread)
 constexpr int kGH = 64;                        // Gauss-Hermite nodes
 constexpr int kMaxJobs = 4;
