@@ -80,3 +80,61 @@ def test_prepare_rejects_bad_arguments_on_host(Q, kw, status):
     with pytest.raises(Q.SeedQError) as e:
         _prepare(Q, **kw)
     assert e.value.status == status
+
+
+@pytest.mark.parametrize("factors,rungs,slopes,rbar,floor_f,status", [
+    ([], [(8, 3), (16, 3)], [1.0], 4.0, 0.06, 1),                              # no tensors
+    ([(4, 12, np.ones(12, np.float32), None)], [(8, 3), (16, 3)], [1.0], 4.0, 0.06, 1),
+    ([(4, 16, np.zeros(16, np.float32), None)], [(8, 3), (16, 3)], [1.0], 4.0, 0.06, 1),
+    ([(4, 16, np.ones(16, np.float32), np.array([1, 0, 1, 1], np.float32))],
+     [(8, 3), (16, 3)], [1.0], 4.0, 0.06, 1),                                  # rho must be > 0
+    ([(4, 16, np.ones(16, np.float32), None)], [(9, 3), (16, 3)], [1.0], 4.0, 0.06, 6),
+    ([(4, 16, np.ones(16, np.float32), None)], [(16, 3), (8, 3)], [1.0], 4.0, 0.06, 3),
+    ([(4, 16, np.ones(16, np.float32), None)], [(8, 3), (16, 3)], [-1.0], 4.0, 0.06, 3),
+    ([(4, 16, np.ones(16, np.float32), None)], [(8, 3), (16, 3)], [1.0], 0.0, 0.06, 1),
+    ([(4, 16, np.ones(16, np.float32), None)], [(8, 3), (16, 3)], [1.0], 4.0, 1.5, 1),
+])
+def test_allocate_rejects_bad_arguments_on_host(Q, factors, rungs, slopes, rbar, floor_f, status):
+    """Alg. 1 on the device validates everything on the host before any CUDA call."""
+    with pytest.raises(Q.SeedQError) as e:
+        Q.allocate(factors, rungs, slopes, rbar, floor_f, stream=0)
+    assert e.value.status == status
+
+
+def _dims(**kw):
+    d = dict(n_layers=1, d_model=64, n_heads=2, n_kv_heads=1, head_dim=32, d_ff=96, vocab=10)
+    d.update(kw)
+    return d
+
+
+@pytest.mark.parametrize("kw", [dict(d_model=48), dict(d_ff=40), dict(n_heads=3, n_kv_heads=2),
+                                dict(n_layers=0), dict(head_dim=20), dict(vocab=0)])
+def test_importance_rejects_bad_shapes_on_host(Q, kw):
+    """Shapes the column pass cannot tile (in-dimensions not multiples of 32,
+    query heads not a multiple of the key-value heads) fail before any launch."""
+    fake = 1 << 20  # 16-byte aligned, never dereferenced: validation comes first
+    layer = {k: fake for k in ("attn_norm", "mlp_norm", "wq", "wk", "wv", "wo", "wgate", "wup", "wdown")}
+    dims = _dims(**kw)
+    out = {k: fake for k in ("a_o", "a_down", "rho_o", "rho_down")}
+    with pytest.raises(Q.SeedQError) as e:
+        Q.importance(dims, [layer] * max(dims["n_layers"], 1), fake, fake, out, stream=0)
+    assert e.value.status == 1
+
+
+def test_importance_rejects_missing_pointers_on_host(Q):
+    fake = 1 << 20
+    layer = {k: fake for k in ("attn_norm", "mlp_norm", "wq", "wk", "wv", "wo", "wgate", "wup", "wdown")}
+    out = {k: fake for k in ("a_o", "a_down", "rho_o", "rho_down")}
+    for missing in ("wv", "attn_norm"):
+        bad = dict(layer)
+        bad[missing] = 0
+        with pytest.raises(Q.SeedQError) as e:
+            Q.importance(_dims(), [bad], fake, fake, out, stream=0)
+        assert e.value.status == 1
+    misaligned = dict(layer, wq=fake + 2)
+    with pytest.raises(Q.SeedQError) as e:
+        Q.importance(_dims(), [misaligned], fake, fake, out, stream=0)
+    assert e.value.status == 1
+    with pytest.raises(Q.SeedQError) as e:
+        Q.importance(_dims(), [layer], fake, fake, dict(out, a_o=0), stream=0)
+    assert e.value.status == 1
