@@ -178,10 +178,12 @@ def test_importance_small_models_against_oracle(Q, G, name):
         assert (names.index(f"l{l}.{k}"), c) in got
 
 
-def test_importance_llama2_7b_shape_sampled(Q, G):
-    """The full Llama-2-7B-shaped checkpoint in the launch configuration of the
-    benchmark; outputs checked on samples the oracle computes one by one."""
-    spec = W.MODELS["llama2_7b"]
+@pytest.mark.parametrize("name", ["llama2_7b", "llama3_8b"])
+def test_importance_full_shape_sampled(Q, G, name):
+    """Full Llama-shaped checkpoints in the launch configuration of the
+    benchmark (Llama-3-8B: 4 query heads per value head); outputs checked on
+    samples the oracle computes one by one."""
+    spec = W.MODELS[name]
     gm = G.synth_model_device(spec)
     out = G.importance_buffers(spec)
     got = G.run_importance(gm, out)
@@ -203,13 +205,15 @@ def test_importance_llama2_7b_shape_sampled(Q, G):
             g2 = I.sq_rows(W.synth_weight_rows(spec, l, "gate", int(c), 1), a_mlp)
             u = I.sq_rows(W.synth_weight_rows(spec, l, "up", int(c), 1), a_mlp)
             assert _rel(a_dn[l, c], I.silu_sq_moment(g2)[0] * u[0]) < ONE_HOP
-    # rho of the last down projection: the head's column sums of squares.
-    head = np.zeros(d)
-    R = spec.vocab
-    for r0 in range(0, R, 4000):
-        head += I.sq_cols(W.synth_weight_rows(spec, None, "lm_head", r0, min(4000, R - r0)),
-                          np.ones(min(4000, R - r0)))
-    assert _rel(r_dn[L - 1], I.unit_mean(head)) < 2 * ONE_HOP
+    # rho of the last down projection: the head's column sums of squares
+    # (checked on the smaller head; the 128k-row one takes minutes on the host).
+    if spec.vocab <= 64000:
+        head = np.zeros(d)
+        R = spec.vocab
+        for r0 in range(0, R, 4000):
+            head += I.sq_cols(W.synth_weight_rows(spec, None, "lm_head", r0, min(4000, R - r0)),
+                              np.ones(min(4000, R - r0)))
+        assert _rel(r_dn[L - 1], I.unit_mean(head)) < 2 * ONE_HOP
     # Planted super weights: exact statistic and selected.
     names = spec.tensor_names()
     dr = out["dyn_range"].cpu().numpy()
