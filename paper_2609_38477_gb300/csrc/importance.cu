@@ -952,7 +952,8 @@ seedq_status launch_cols(ColArgs &A, const ColScratch &S, cudaStream_t st) {
   if (items > S.part_cap || tiles > S.arrive_cap) return SEEDQ_ERR_INVALID_ARG;
   if (items == 0) return SEEDQ_OK;
   A.items = (int32_t)items;
-  static const cudaError_t attr = cudaFuncSetAttribute(
+  // Per call: the attribute belongs to the current device.
+  const cudaError_t attr = cudaFuncSetAttribute(
       k_colpass, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kRingBytes);
   if (attr != cudaSuccess) return cuda_fail(attr);
   k_colpass<<<(int)std::min<int64_t>(items, S.ctas), kCT, kRingBytes, st>>>(A, S.ghist);
