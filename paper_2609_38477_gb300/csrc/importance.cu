@@ -136,12 +136,12 @@ __device__ __forceinline__ double half_val(uint32_t bits) {
 // Median filter.  The dynamic-range statistic reaches 1e3 only when the
 // column median is below max / 1e3.  Each row slab takes a provisional
 // maximum M0_s from its first 512 rows and a threshold U0_s >= 2.01 K M0_s /
-// 1e3 (K = 16), and counts |W| < U0_s while it streams.  With M0 = min_s M0_s
-// (whose threshold U0 is the smallest), if the column maximum M <= K M0 and
-// the counts sum to at most (R-1)/2, then at most (R-1)/2 elements lie below
-// U0 (the counts are FP16 compares of FP16 magnitudes, exact), both middle order statistics are >= U0, and max / (median + eps) <=
-// 1e3 / 2.01: the column cannot qualify.  Every other column gets its exact
-// median.
+// 1e3 (K = 16), and counts |W| < U0_s while it streams (FP16 compares of FP16
+// magnitudes, counted exactly).  With M0 = min_s M0_s, whose threshold U0 is
+// the smallest, the counts bound the number of elements below U0.  If the
+// column maximum M <= K M0 and the counts sum to at most (R-1)/2, both middle
+// order statistics are >= U0, so max / (median + eps) <= 1e3 / 2.01: the
+// column cannot qualify.  Every other column gets its exact median.
 constexpr float kGrowth = 16.f;
 constexpr float kLowFrac = 2.01f * kGrowth / 1000.f;
 
@@ -197,7 +197,9 @@ __device__ __forceinline__ void stage_rows(const uint4 *slot, const float *wst, 
 template <bool kCols, bool kRows>
 __device__ __forceinline__ void stage_dispatch(const uint4 *slot, const float *wst, bool ones,
                                                int nu, float *rowpart, Acc &A) {
-  if (nu == kUnroll) {
+  // The full-mask path only when every lane of the warp has all 8 rows (row
+  // counts that are not multiples of 64 leave the last stage ragged).
+  if (__all_sync(0xffffffffu, nu == kUnroll)) {
     if (ones) stage_rows<kCols, kRows, true, true>(slot, wst, nu, rowpart, A);
     else stage_rows<kCols, kRows, false, true>(slot, wst, nu, rowpart, A);
   } else {

@@ -312,6 +312,9 @@ MODELS = {
                       "2 layers, d 256, 4 query / 2 key-value heads of 64, d_ff 640, vocab 300"),
     "tiny_mha": ModelSpec("tiny_mha", 3, 256, 4, 4, 64, 512, 272, 37,
                           "3 layers, d 256, 4 heads of 64 (no sharing), d_ff 512, vocab 272"),
+    "tiny_odd": ModelSpec("tiny_odd", 2, 160, 5, 1, 32, 96, 77, 47,
+                          "2 layers, d 160, 5 query heads of 32 sharing 1 key-value head, "
+                          "d_ff 96, vocab 77 (row counts not multiples of 64)"),
     "llama2_7b": ModelSpec("llama2_7b", 32, 4096, 32, 32, 128, 11008, 32000, 41,
                            "Llama-2-7B-shaped: 32 layers, d 4096, 32 heads of 128, d_ff 11008, "
                            "vocab 32000, FP16"),

@@ -170,7 +170,7 @@ def _check_model(Q, G, name):
     return spec, got_out
 
 
-@pytest.mark.parametrize("name", ["tiny", "tiny_mha"])
+@pytest.mark.parametrize("name", ["tiny", "tiny_mha", "tiny_odd"])
 def test_importance_small_models_against_oracle(Q, G, name):
     spec, got = _check_model(Q, G, name)
     names = spec.tensor_names()
