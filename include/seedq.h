@@ -244,7 +244,9 @@ seedq_status seedq_encode_blocks(int32_t S, int32_t k, const float *w, int64_t n
 /* Every block of a prepared layer at the rung its plan assigns: W is device
  * R x C float32 in the original column order (block (r, c) holds the columns
  * perm[8c .. 8c+7] of row r); outputs have R x (C/8) entries in row-major
- * block order. */
+ * block order.  The layer's outlier columns enter the search as zero: their
+ * FP16 values overwrite the decoded columns (Sec. 3.5), and a spike left in
+ * place would distort its seven block-mates. */
 seedq_status seedq_encode_layer(const seedq_layer *layer, const float *W, uint32_t *seed,
                                 int8_t *E, int8_t *t, double *err, void *cuda_stream);
 

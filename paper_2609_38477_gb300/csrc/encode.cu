@@ -352,7 +352,15 @@ __global__ void __launch_bounds__(kEncWarps * 32) k_encode_layer(const __grid_co
     const int g = rung_of(bk, p.J, c);
     float wv[8];
 #pragma unroll
-    for (int i = 0; i < 8; ++i) wv[i] = __ldg(W + r * p.C + __ldg(p.perm + 8 * c + i));
+    for (int i = 0; i < 8; ++i) {
+      const int col = __ldg(p.perm + 8 * c + i);
+      // Outlier columns are stored in FP16 and overwrite the decode (Sec. 3.5):
+      // the search sees them as zero, so their spike does not leak into the
+      // block-mates.
+      bool outlier = false;
+      for (int o = 0; o < p.n_out; ++o) outlier |= (p.out_cols[o] == col);
+      wv[i] = outlier ? 0.f : __ldg(W + r * p.C + col);
+    }
     encode_dispatch(rung_S(p.code[g]), rung_K(p.code[g]), tabs + (size_t)p.slot[g] * 512, wv, lane, o, blk);
   }
 }
