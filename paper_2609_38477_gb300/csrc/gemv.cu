@@ -101,31 +101,35 @@ __device__ __forceinline__ int cta_of(const int64_t *cb, int ctas, int64_t u) {
 
 // One block: reconstruct its 8 weights and add scale * sum_i I_i x_b[i] to
 // acc[b].  xc holds the block's activations weight-major, NB per weight
-// (xc[i * NB + b]).  Per batch column the products form two chains (weights
-// 0-3 and 4-7); at NB >= 2 two batch columns share each packed instruction.
+// (xc[i * NB + b]).  At NB = 1 the products run in the packed halves the
+// reconstruction leaves them in (even and odd weights); at NB >= 2 two batch
+// columns share each packed instruction, in two chains (weights 0-3, 4-7).
 template <int K, int NB>
 __device__ __forceinline__ void block_fma(const uint32_t (&w)[3], uint32_t sh, const uint64_t *tab,
                                           const RungRt<K> &rc, const float *xc, float (&acc)[NB]) {
   const uint32_t lo = __funnelshift_r(w[0], w[1], sh);
   const uint32_t hi = __funnelshift_r(w[1], w[2], sh);
-  float I[8], scale;
-  reconstruct_rt<K>(lo, hi, tab, rc, I, scale);
+  uint64_t I2[4];
+  float scale;
+  reconstruct_rt2<K>(lo, hi, tab, rc, I2, scale);
   if constexpr (NB == 1) {
-    const float4 x0 = *reinterpret_cast<const float4 *>(xc);
-    const float4 x1 = *reinterpret_cast<const float4 *>(xc + 4);
-    float s0 = I[0] * x0.x, s1 = I[4] * x1.x;
-    s0 = __fmaf_rn(I[1], x0.y, s0);
-    s1 = __fmaf_rn(I[5], x1.y, s1);
-    s0 = __fmaf_rn(I[2], x0.z, s0);
-    s1 = __fmaf_rn(I[6], x1.z, s1);
-    s0 = __fmaf_rn(I[3], x0.w, s0);
-    s1 = __fmaf_rn(I[7], x1.w, s1);
-    acc[0] = __fmaf_rn(scale, s0 + s1, acc[0]);
+    const ulonglong2 xa = *reinterpret_cast<const ulonglong2 *>(xc);
+    const ulonglong2 xb = *reinterpret_cast<const ulonglong2 *>(xc + 4);
+    uint64_t s2 = f2_mul(I2[0], xa.x);
+    s2 = f2_fma(I2[1], xa.y, s2);
+    s2 = f2_fma(I2[2], xb.x, s2);
+    s2 = f2_fma(I2[3], xb.y, s2);
+    const float2 sv = f2_unpack(s2);
+    acc[0] = __fmaf_rn(scale, sv.x + sv.y, acc[0]);
   } else {
     const uint64_t *x2 = reinterpret_cast<const uint64_t *>(xc);  // pairs of batch columns
     uint64_t Ip[8];
 #pragma unroll
-    for (int i = 0; i < 8; ++i) Ip[i] = f2_pack(I[i], I[i]);
+    for (int p = 0; p < 4; ++p) {
+      const float2 v = f2_unpack(I2[p]);
+      Ip[2 * p] = f2_pack(v.x, v.x);
+      Ip[2 * p + 1] = f2_pack(v.y, v.y);
+    }
     const uint64_t sp = f2_pack(scale, scale);
 #pragma unroll
     for (int q = 0; q < NB / 2; ++q) {

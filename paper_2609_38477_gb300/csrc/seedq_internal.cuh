@@ -5,6 +5,7 @@
 #include <stdint.h>
 
 #include "../../include/seedq.h"
+#include "f32x2.cuh"
 
 namespace seedq {
 
@@ -261,9 +262,13 @@ __device__ __forceinline__ uint32_t qwin3(uint32_t q0, uint32_t q1, uint32_t q2)
   else return __funnelshift_r(q1, q2, N - 32);
 }
 
-template <int K, int I, int J>
-__device__ __forceinline__ float state_chain_rt(uint32_t q0, uint32_t q1, uint32_t q2,
-                                                const RungRt<K> &rc, const float (&tf)[K], float acc) {
+// The chains of weights 2p and 2p + 1 run side by side in the two halves of
+// packed f32x2 FMAs (each half rounds as the scalar FMA would, so I is the
+// same exact integer).
+template <int K, int P, int J>
+__device__ __forceinline__ uint64_t state_chain2(uint32_t q0, uint32_t q1, uint32_t q2,
+                                                 const RungRt<K> &rc, const uint64_t (&tf2)[K],
+                                                 uint64_t acc) {
   if constexpr (J < 0) {
     return acc;
   } else {
@@ -271,26 +276,20 @@ __device__ __forceinline__ float state_chain_rt(uint32_t q0, uint32_t q1, uint32
     constexpr int grp = (K - 1 - J) / G;
     constexpr int jt = K - 1 - grp * G;
     constexpr int d = jt - J;
-    const uint32_t win = qwin3<I * K + jt>(q0, q1, q2);
-    acc = __fmaf_rn(tf[J], __uint_as_float(lop_and_or(win, rc.s_msk[d], rc.s_exp[d])), acc);
-    return state_chain_rt<K, I, J - 1>(q0, q1, q2, rc, tf, acc);
+    const uint32_t w0 = qwin3<(2 * P) * K + jt>(q0, q1, q2);
+    const uint32_t w1 = qwin3<(2 * P + 1) * K + jt>(q0, q1, q2);
+    const uint64_t st = f2_pack(__uint_as_float(lop_and_or(w0, rc.s_msk[d], rc.s_exp[d])),
+                                __uint_as_float(lop_and_or(w1, rc.s_msk[d], rc.s_exp[d])));
+    acc = f2_fma(tf2[J], st, acc);
+    return state_chain2<K, P, J - 1>(q0, q1, q2, rc, tf2, acc);
   }
 }
 
-template <int K, int I>
-__device__ __forceinline__ void weights_from_rt(uint32_t q0, uint32_t q1, uint32_t q2,
-                                                const RungRt<K> &rc, const float (&tf)[K],
-                                                float init, float (&Iv)[8]) {
-  if constexpr (I < 8) {
-    Iv[I] = state_chain_rt<K, I, K - 1>(q0, q1, q2, rc, tf, init);
-    weights_from_rt<K, I + 1>(q0, q1, q2, rc, tf, init, Iv);
-  }
-}
-
-// lo, hi: the block's 64 field bits starting at its first bit.
+// lo, hi: the block's 64 field bits starting at its first bit.  Ip[p] holds
+// (I[2p], I[2p + 1]).
 template <int K>
-__device__ __forceinline__ void reconstruct_rt(uint32_t lo, uint32_t hi, const uint64_t *tab,
-                                               const RungRt<K> &rc, float (&I)[8], float &scale) {
+__device__ __forceinline__ void reconstruct_rt2(uint32_t lo, uint32_t hi, const uint64_t *tab,
+                                                const RungRt<K> &rc, uint64_t (&Ip)[4], float &scale) {
   // For S = 8 the second table half is all zero, so both lookups are always valid.
   const uint64_t Q = tab[lo & 255u] ^ tab[256 + __byte_perm(lo, 0, 0x4441)];
   const uint32_t qlo = (uint32_t)Q, qhi = (uint32_t)(Q >> 32);
@@ -301,6 +300,7 @@ __device__ __forceinline__ void reconstruct_rt(uint32_t lo, uint32_t hi, const u
   const uint32_t e8 = lop_and_xor(f, rc.e_msk, rc.e_x);
   scale = __uint_as_float(e8 * (1u << 23) + rc.sc);
   float tf[K];
+  uint64_t tf2[K];
   uint32_t f2 = 0;
   if constexpr (K > 4) f2 = f >> 16;
 #pragma unroll
@@ -308,11 +308,29 @@ __device__ __forceinline__ void reconstruct_rt(uint32_t lo, uint32_t hi, const u
     const int P = (4 + 4 * j <= 19) ? 4 + 4 * j : 4 + 4 * j - 16;
     const uint32_t w = (4 + 4 * j <= 19) ? f : f2;
     tf[j] = __uint_as_float(lop_and_xor(w, rc.t_msk[j], rc.t_x[j])) - (float)((1 << (23 - P)) + 8);
+    tf2[j] = f2_pack(tf[j], tf[j]);
   }
   float init = 0.f;
 #pragma unroll
   for (int j = 0; j < K; ++j) init = __fmaf_rn(tf[j], rc.cinit[j], init);
-  weights_from_rt<K, 0>(q0, q1, q2, rc, tf, init, I);
+  const uint64_t init2 = f2_pack(init, init);
+  Ip[0] = state_chain2<K, 0, K - 1>(q0, q1, q2, rc, tf2, init2);
+  Ip[1] = state_chain2<K, 1, K - 1>(q0, q1, q2, rc, tf2, init2);
+  Ip[2] = state_chain2<K, 2, K - 1>(q0, q1, q2, rc, tf2, init2);
+  Ip[3] = state_chain2<K, 3, K - 1>(q0, q1, q2, rc, tf2, init2);
+}
+
+template <int K>
+__device__ __forceinline__ void reconstruct_rt(uint32_t lo, uint32_t hi, const uint64_t *tab,
+                                               const RungRt<K> &rc, float (&I)[8], float &scale) {
+  uint64_t Ip[4];
+  reconstruct_rt2<K>(lo, hi, tab, rc, Ip, scale);
+#pragma unroll
+  for (int p = 0; p < 4; ++p) {
+    const float2 v = f2_unpack(Ip[p]);
+    I[2 * p] = v.x;
+    I[2 * p + 1] = v.y;
+  }
 }
 
 
