@@ -235,10 +235,11 @@ __device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t 
     const int cs = pcs[pi].ca + t * CF::ST, ce = min(pcs[pi].cb, cs + CF::ST);
     const int64_t r0 = pcs[pi].g * 32;
     const int64_t ridx = r0 + lane;
-    const int64_t row = __ldg(p.rowperm + (ridx < p.R ? ridx : r0));
-    const uint64_t roff = __ldg(p.row_off + row);
+    const uint4 *rec = p.rowrec + 2 * (ridx < p.R ? ridx : r0);
+    const uint4 m0 = __ldg(rec), m1 = __ldg(rec + 1);
+    const uint64_t roff = (uint64_t)m0.x | ((uint64_t)m0.y << 32);
     int16_t *mybk = bk + (sb * 32 + lane) * 8;
-    for (int j = 0; j < J - 1; ++j) mybk[j] = __ldg(p.brk + row * (J - 1) + j);
+    *reinterpret_cast<uint4 *>(mybk) = make_uint4(m0.z, m0.w, m1.x, m1.y);
     const uint64_t bit_cs = roff + lane_bits_before(mybk, J, p.L, nb, cs);
     const uint64_t b_lo = (bit_cs >> 3) & ~(uint64_t)15;
     uint64_t b_hi = (roff + lane_bits_before(mybk, J, p.L, nb, ce) + 96 + 7) >> 3;

@@ -93,6 +93,25 @@ __global__ void k_iota(int64_t n, int32_t *__restrict__ out) {
     out[i] = (int32_t)i;
 }
 
+// The fused kernel's per-row record, in its row order: row r = rowperm[i] at
+// position i, with its bit offset and breakpoints in two 16-byte words, so a
+// warp fetches its 32 rows' plan data with two contiguous loads per lane.
+__global__ void k_rowrec(const int32_t *__restrict__ rowperm, const uint64_t *__restrict__ row_off,
+                         const int32_t *__restrict__ brk, int J, int64_t R, uint4 *__restrict__ rec) {
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < R;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t r = rowperm[i];
+    const uint64_t off = row_off[r];
+    static_assert(kMaxJ == 9, "the record holds eight breakpoints");
+    uint32_t b[kMaxJ - 1];
+#pragma unroll
+    for (int j = 0; j < kMaxJ - 1; ++j)
+      b[j] = j < J - 1 ? (uint32_t)(uint16_t)brk[r * (J - 1) + j] : 0u;
+    rec[2 * i] = make_uint4((uint32_t)off, (uint32_t)(off >> 32), b[0] | (b[1] << 16), b[2] | (b[3] << 16));
+    rec[2 * i + 1] = make_uint4(b[4] | (b[5] << 16), b[6] | (b[7] << 16), 0u, 0u);
+  }
+}
+
 __global__ void k_invperm(const int32_t *__restrict__ perm, int C, int32_t *__restrict__ inv) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i < C) inv[perm[i]] = i;
@@ -343,6 +362,7 @@ static void free_layer(seedq_layer *L) {
   cudaFree(L->d_flags);
   cudaFree(L->d_summary);
   cudaFree(L->d_rowperm);
+  cudaFree(L->d_rowrec);
   cudaFree(L->d_counters);
   cudaFree(L->d_slots);
   cudaFree(L->d_xperm);
@@ -585,6 +605,7 @@ seedq_status seedq_layer_prepare(const seedq_layer_desc *d, const seedq_schedule
   }
   const int64_t ngroups = (R + 31) / 32;
   ALLOC(L->d_rowperm, sizeof(int32_t) * R);
+  ALLOC(L->d_rowrec, sizeof(uint4) * 2 * R);
   ALLOC(L->d_counters, sizeof(int32_t) * ngroups);
   ALLOC(L->d_slots, sizeof(float) * L->max_ctas * 2 * 32 * kMaxBatch);
   // Weight-major activations, padded to the kernel's batch template.
@@ -594,6 +615,7 @@ seedq_status seedq_layer_prepare(const seedq_layer_desc *d, const seedq_schedule
 #undef ALLOC
   L->args.perm = L->d_perm;
   L->args.rowperm = L->d_rowperm;
+  L->args.rowrec = L->d_rowrec;
   L->args.counters = L->d_counters;
   L->args.slots = L->d_slots;
   L->args.xperm = L->d_xperm;
@@ -638,6 +660,8 @@ seedq_status seedq_layer_prepare(const seedq_layer_desc *d, const seedq_schedule
     } else {
       k_rowrank<<<(int)((R + 255) / 256), 256, 0, st>>>(L->d_rho, (int)R, L->d_rowperm);
     }
+    k_rowrec<<<(int)((R + 255) / 256 < 4096 ? (R + 255) / 256 : 4096), 256, 0, st>>>(
+        L->d_rowperm, L->d_row_off, L->d_brk, J, R, L->d_rowrec);
     if (e == cudaSuccess) e = cudaMemsetAsync(L->d_counters, 0, sizeof(int32_t) * ngroups, st);
     if (e == cudaSuccess) e = cudaGetLastError();
   }

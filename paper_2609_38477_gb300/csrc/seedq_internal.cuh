@@ -36,6 +36,9 @@ struct LayerArgs {
   const int32_t *invperm;   // C: position of column j in the permuted order
   const uint16_t *out_vals; // R x n_out binary16
   const int32_t *rowperm;   // R: order in which rows are grouped 32 to a warp
+  const uint4 *rowrec;      // R x 2, at row position i (row rowperm[i]): its bit
+                            // offset (words 0-1) and its breakpoints as int16
+                            // pairs (words 2-5, zero past J - 1)
   float *xperm;             // C x n: activations in permuted order, weight-major
   int32_t *counters;        // row groups: arrivals of partial sums (0 between calls)
   float *slots;             // max_ctas x 2 x 32 x 16 partial sums of row groups
@@ -86,6 +89,7 @@ struct seedq_layer {
   int32_t *d_brk;
   int32_t *d_tcnt;
   int32_t *d_rowperm;
+  uint4 *d_rowrec;
   int32_t *d_counters;
   float *d_slots;
   float *d_xperm;
