@@ -188,17 +188,21 @@ __device__ __forceinline__ void dispatch_cols(int code, const uint32_t *rowbuf, 
   }
 }
 
-// Bits of the lane's row before block x (rung j spans [bk[j-1], bk[j])).
-__device__ __forceinline__ uint32_t lane_bits_before(const int16_t *bk, int J, const int32_t *L,
-                                                     int nb, int x) {
-  uint32_t s = 0;
-  int lo = 0;
-  for (int j = 0; j < J; ++j) {
-    const int hi = (j < J - 1) ? bk[j] : nb;
-    s += (uint32_t)L[j] * (uint32_t)(min(max(x, lo), hi) - lo);
-    lo = hi;
+// Bits of the lane's row before blocks cs and ce.  Rung j spans blocks
+// [bk[j-1], bk[j]) and the breakpoints rise along the row, so the bits before
+// block x are L[0] x plus, for every breakpoint below x, the rate step dL[j]
+// times the blocks past it.  bw: the row's breakpoints as int16 pairs (zero
+// past J - 1, where dL is zero).
+__device__ __forceinline__ void lane_bits_before(const uint32_t (&bw)[4], const LayerArgs &p, int cs,
+                                                 int ce, uint32_t &s_cs, uint32_t &s_ce) {
+  s_cs = (uint32_t)p.L[0] * (uint32_t)cs;
+  s_ce = (uint32_t)p.L[0] * (uint32_t)ce;
+#pragma unroll
+  for (int j = 0; j < kMaxJ - 1; ++j) {
+    const int b = (int)((bw[j >> 1] >> (16 * (j & 1))) & 0xffffu);
+    s_cs += (uint32_t)p.dL[j] * (uint32_t)max(cs - b, 0);
+    s_ce += (uint32_t)p.dL[j] * (uint32_t)max(ce - b, 0);
   }
-  return s;
 }
 
 // A piece of a round: blocks [ca, cb) of row group g of the round's tensor.
@@ -240,9 +244,12 @@ __device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t 
     const uint64_t roff = (uint64_t)m0.x | ((uint64_t)m0.y << 32);
     int16_t *mybk = bk + (sb * 32 + lane) * 8;
     *reinterpret_cast<uint4 *>(mybk) = make_uint4(m0.z, m0.w, m1.x, m1.y);
-    const uint64_t bit_cs = roff + lane_bits_before(mybk, J, p.L, nb, cs);
+    const uint32_t bw[4] = {m0.z, m0.w, m1.x, m1.y};
+    uint32_t s_cs, s_ce;
+    lane_bits_before(bw, p, cs, ce, s_cs, s_ce);
+    const uint64_t bit_cs = roff + s_cs;
     const uint64_t b_lo = (bit_cs >> 3) & ~(uint64_t)15;
-    uint64_t b_hi = (roff + lane_bits_before(mybk, J, p.L, nb, ce) + 96 + 7) >> 3;
+    uint64_t b_hi = (roff + s_ce + 96 + 7) >> 3;
     b_hi = (b_hi + 15) & ~(uint64_t)15;
     if (b_hi > T.stream_bytes) b_hi = T.stream_bytes & ~(uint64_t)15;
     const int npc = b_hi > b_lo ? (int)min((uint64_t)CF::PIECES, (b_hi - b_lo) >> 4) : 0;

@@ -556,6 +556,7 @@ seedq_status seedq_layer_prepare(const seedq_layer_desc *d, const seedq_schedule
     L->args.slot[j] = (L->S[j] - 8) / 2;
     if (j + 1 < J) L->theta[j] = s->theta[j];
   }
+  for (int j = 0; j < kMaxJ - 1; ++j) L->args.dL[j] = j + 1 < J ? L->args.L[j + 1] - L->args.L[j] : 0;
   L->args.nslots = nslots;
   L->args.n_out = d->n_outliers;
   for (int o = 0; o < d->n_outliers; ++o) L->args.out_cols[o] = d->outlier_cols[o];

@@ -47,6 +47,7 @@ struct LayerArgs {
   int32_t nb;               // C / 8 blocks per row
   int32_t J;
   int32_t L[kMaxJ];         // block bits per rung
+  int32_t dL[kMaxJ - 1];    // L[j + 1] - L[j] for j < J - 1, else 0
   int32_t code[kMaxJ];      // rung_code per rung
   int32_t slot[kMaxJ];      // LFSR table slot per rung
   int32_t nslots;
