@@ -178,25 +178,31 @@ def dist_barrier():
 def algorithmic_counts(w, gts, sched, n):
     """Per-step algorithmic work: warp-instructions of the issue model
     (per weight: k_b LFSR states, k_b integer MACs, one convert, n FMAs) and
-    HBM bytes (payload, plan rows read, x, y)."""
+    HBM bytes (payload, plan rows read, x, y); also the mean k_b and the
+    blocks at each rung."""
     import numpy as np
 
     rungs = sched["rungs"]
     J = len(rungs)
     warp_inst, bytes_, ksum, blocks = 0.0, 0, 0, 0
+    per_rung = np.zeros(J, np.int64)
     for gt in gts:
         t = gt.spec
         rm = gt.layer.rung_map()
         cnt = np.bincount(rm.ravel(), minlength=J)
+        per_rung += cnt[:J]
         for j, (S, k) in enumerate(rungs):
             warp_inst += cnt[j] * 8 * (2 * k + 1 + n) / 32.0
             ksum += int(cnt[j]) * k
         blocks += int(cnt.sum())
         bytes_ += (gt.bits + 7) // 8 + t.R * (8 + 4 * (J - 1)) + 2 * n * t.C + 4 * n * t.R
-    return warp_inst, bytes_, ksum / blocks
+    hist = {f"{S},{k}": int(c) for (S, k), c in zip(rungs, per_rung)}
+    return warp_inst, bytes_, ksum / blocks, hist
 
 
-def traffic_per_launch(kernel_hash: str):
+def traffic_per_launch(kernel_hash: str, workload: str, batch: int):
+    """DRAM bytes of one fused launch from the stored ncu capture, or None when
+    the capture is of another kernel source, workload or batch size."""
     path = os.path.join(ROOT, "profiles", "k_gemv_c1_dram_traffic.txt")
     if not os.path.exists(path):
         return None
@@ -206,6 +212,8 @@ def traffic_per_launch(kernel_hash: str):
             k, v = line.strip().split("=", 1)
             kv[k.strip()] = v.strip()
     if kv.get("kernel_source_sha256") != kernel_hash:
+        return None
+    if kv.get("workload") != workload or kv.get("batch") != str(batch):
         return None
     try:
         return float(kv["dram_bytes_per_launch"])
@@ -413,7 +421,7 @@ def our_arm(args):
 
     mean_step = dist_max(statistics.mean(step_ms))
     mean_e2e = dist_max(statistics.mean(e2e_ms))
-    warp_inst, alg_bytes, mean_k = algorithmic_counts(w, gts, sched, n)
+    warp_inst, alg_bytes, mean_k, rung_hist = algorithmic_counts(w, gts, sched, n)
     call_ms = [statistics.mean(v) for v in per_call]
     kern_ms = statistics.mean(step_ms)  # the step is the fused launches themselves
     props = torch.cuda.get_device_properties(local)
@@ -436,6 +444,7 @@ def our_arm(args):
             "workload": f"{w.name}: {w.description}", "batch": n,
             "bits_per_weight": sched["mean_bits_per_weight"], "weights": w.weights,
             "stream_bytes": stream_bytes, "mean_k": round(mean_k, 4),
+            "blocks_per_rung": rung_hist,
             "l2": f"flushed between timed steps ({FLUSH_BYTES >> 20} MiB write)",
             "parallelism": "replicas" if world > 1 else "single GPU",
         },
@@ -448,7 +457,7 @@ def our_arm(args):
         "roofline": {
             "bound": "alu", "achieved": achieved_issue, "peak": issue_peak,
             "unit": "Gwarp-inst/s", "frac": achieved_issue / issue_peak,
-            "traffic": traffic_per_launch(kernel_source_hash()),
+            "traffic": traffic_per_launch(kernel_source_hash(), w.name, n),
             "kernel": "k_gemv over all tensors of the step in one launch (with its x-permutation pre-kernel)",
             "peak_basis": f"4 warp-inst/clk/SM x {sms} SMs x {sm_max:.0f} MHz",
             "hbm": {"achieved_gbs": achieved_hbm, "peak_gbs": hbm_peak,
