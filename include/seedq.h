@@ -146,13 +146,16 @@ seedq_status seedq_decode_rows(const seedq_layer *layer, int64_t row0,
 /* y = W_hat x (the matrix-vector product the reconstructed weights feed,
  * Sec. 1 and App. C; W_hat is never materialized).  x: device, C bfloat16
  * values (bit patterns) in the original column order; y: device, R float32.
- * Accumulation in fp32. */
+ * Accumulation in fp32.  Errors: INVALID_ARG (NULL layer, x or y), STREAM (no
+ * stream bound), CUDA (launch failed). */
 seedq_status seedq_gemv(const seedq_layer *layer, const uint16_t *x, float *y,
                         void *cuda_stream);
 
 /* Y = X W_hat^T for n = 1..max_batch activation columns: X device n x C
  * bfloat16 row-major, Y device n x R float32 row-major (row b of Y is
- * W_hat x_b).  Each block is reconstructed once and used for all n columns. */
+ * W_hat x_b).  Each block is reconstructed once and used for all n columns.
+ * Errors: INVALID_ARG (NULL pointer, n outside 1..max_batch), STREAM (no
+ * stream bound), CUDA. */
 seedq_status seedq_gemm_small_batch(const seedq_layer *layer, const uint16_t *X,
                                     int32_t n, float *Y, void *cuda_stream);
 
@@ -165,7 +168,9 @@ seedq_status seedq_gemm_small_batch(const seedq_layer *layer, const uint16_t *X,
  * (gemv, gemm_small_batch, gemm_multi) use per-layer scratch (permuted
  * activations, partial sums of row groups cut between SMs), so calls that
  * involve the same layer must not run concurrently on different CUDA
- * streams. */
+ * streams.  Errors: INVALID_ARG (count outside 1..8, a NULL layer, X[i] or
+ * Y[i], n above some layer's max_batch), STREAM (a layer without a bound
+ * stream), CUDA. */
 seedq_status seedq_gemm_multi(const seedq_layer *const *layers, int32_t count,
                               const uint16_t *const *X, int32_t n, float *const *Y,
                               void *cuda_stream);
@@ -185,27 +190,37 @@ seedq_status seedq_gemm_multi(const seedq_layer *const *layers, int32_t count,
  * layers' scratch, so they must not overlap with other calls on those layers. */
 typedef struct seedq_layer_set seedq_layer_set;
 
-/* count: 1..65535 layers, each bound; max_batch of the set = the smallest. */
+/* count: 1..65535 layers, each bound; max_batch of the set = the smallest.
+ * Errors: INVALID_ARG (NULL array or entry, count out of range), STREAM (a
+ * layer without a bound stream), NOMEM, CUDA. */
 seedq_status seedq_layer_set_create(const seedq_layer *const *layers, int32_t count,
                                     seedq_layer_set **out);
-/* Host arrays of count + 1 entries each (either may be NULL). */
+/* Host arrays of count + 1 entries each (either may be NULL).  Errors:
+ * INVALID_ARG (NULL set). */
 seedq_status seedq_layer_set_layout(const seedq_layer_set *set, int64_t *col_offsets,
                                     int64_t *row_offsets);
-/* Y_i = X_i W_hat_i^T for every tensor of the set, n = 1..max_batch. */
+/* Y_i = X_i W_hat_i^T for every tensor of the set, n = 1..max_batch (the
+ * tensors are independent, Alg. 2; any order, Sec. 3.6).  Asynchronous like
+ * the other hot calls.  Errors: INVALID_ARG (NULL set, X or Y, n out of
+ * range), CUDA. */
 seedq_status seedq_gemm_set(const seedq_layer_set *set, const uint16_t *X, int32_t n, float *Y,
                             void *cuda_stream);
 seedq_status seedq_layer_set_release(seedq_layer_set *set);
 
-/* Host copy of the rung index (0..J-1) of blocks of rows [row0, row0+nrows):
- * rungs_host receives nrows x (C/8) bytes.  Synchronous. */
+/* Introspection for parity tests (the plan of Alg. 2 as the kernels hold it).
+ * Host copy of the rung index (0..J-1) of blocks of rows [row0, row0+nrows):
+ * rungs_host receives nrows x (C/8) bytes.  Synchronous.  Errors:
+ * INVALID_ARG (NULL pointer, rows out of range), NOMEM, CUDA. */
 seedq_status seedq_layer_rung_map(const seedq_layer *layer, int64_t row0,
                                   int64_t nrows, uint8_t *rungs_host);
 
-/* Host copy of the column permutation (C int32): block c of a row holds
- * original columns perm[8c .. 8c+7].  Synchronous. */
+/* Host copy of the column permutation (C int32, Sec. 3.3): block c of a row
+ * holds original columns perm[8c .. 8c+7].  Synchronous.  Errors: INVALID_ARG
+ * (NULL pointer), CUDA. */
 seedq_status seedq_layer_perm(const seedq_layer *layer, int32_t *perm_host);
 
-/* Host copy of the per-row bit offsets (R+1 uint64, offsets[R] = total). */
+/* Host copy of the per-row bit offsets (R+1 uint64, offsets[R] = total).
+ * Synchronous.  Errors: INVALID_ARG (NULL pointer), CUDA. */
 seedq_status seedq_layer_row_offsets(const seedq_layer *layer, uint64_t *offsets_host);
 
 /* Device error flags accumulated by the layer's kernels since prepare (bit 0:
@@ -289,7 +304,8 @@ typedef struct {
 
 typedef struct seedq_container seedq_container;
 
-/* Write the schedule and ntensors tensors to path (replacing the file). */
+/* Write the schedule and ntensors tensors to path (replacing the file).
+ * Errors: INVALID_ARG (NULL or inconsistent schedule or tensor fields), IO. */
 seedq_status seedq_container_write(const char *path, const seedq_schedule *sched,
                                    int32_t ntensors, const seedq_container_tensor *tensors);
 /* Read and validate a container; *out receives it (release with _close).
@@ -307,7 +323,9 @@ seedq_status seedq_container_close(seedq_container *c);
  * state `key` and uses seed = 1 + (h>>32) mod (2^S-1), E = -8 + ((h>>24)&255)
  * mod 6, t_j = ((h>>4j)&15) - 8 at the rung the plan assigns.  stream: device,
  * stream_bytes >= seedq_stream_bytes_required(plan bits); zeroed first.  A
- * benchmark and test input generator, not part of the paper's method. */
+ * benchmark and test input generator, not part of the paper's method.
+ * Synchronous.  Errors: INVALID_ARG (NULL layer or stream, stream not 16-byte
+ * aligned), STREAM (buffer too small), CUDA. */
 seedq_status seedq_synth_stream(const seedq_layer *layer, uint64_t key,
                                 void *stream, uint64_t stream_bytes,
                                 void *cuda_stream);
