@@ -188,6 +188,50 @@ def test_stored_rho_is_the_proxy_at_unit_mean():
             assert abs(float(np.mean(got.astype(np.float64))) - 1.0) < 1e-6
 
 
+@pytest.mark.parametrize("name", ["tiny", "tiny_mha", "tiny_odd"])
+def test_importance_tables_wiring(name):
+    """Each tensor's entry carries the factors of its own inputs: q, k, v read
+    the attention norm's gain, gate and up the MLP norm's, the head the final
+    norm's (Eq. gamma, squared gains decoded here from the FP16 bits without
+    numpy); o takes the second moment of W_v's outputs repeated over the query
+    heads and down the gate/up propagation of the MLP gain (Eq. prop, the
+    formulas pinned above by sampling); only o and down carry rho."""
+    import struct
+
+    m = W.SynthModel(W.MODELS[name])
+    s = m.spec
+    tables = I.importance_tables(m)
+    assert len(tables) == 7 * s.n_layers + 1
+
+    def sq_gain(bits):
+        vals = struct.unpack("<%de" % len(bits), np.asarray(bits, np.uint16).tobytes())
+        return np.array([v * v for v in vals], np.float64)
+
+    for l in range(s.n_layers):
+        ga, gm = sq_gain(m.gain(l, "attn")), sq_gain(m.gain(l, "mlp"))
+        names = [t[0] for t in tables[7 * l: 7 * l + 7]]
+        assert names == [f"l{l}.{k}" for k in I.KINDS]
+        for j in (0, 1, 2):
+            assert np.array_equal(tables[7 * l + j][1], ga.astype(np.float32)), (l, j)
+        for j in (4, 5):
+            assert np.array_equal(tables[7 * l + j][1], gm.astype(np.float32)), (l, j)
+        Wv = I.f16(m.weight(l, "v"))
+        vo = (Wv * Wv) @ ga
+        hd = s.head_dim
+        rep = s.n_heads // s.n_kv_heads
+        ao = np.concatenate([vo[(h // rep) * hd:(h // rep + 1) * hd] for h in range(s.n_heads)])
+        assert np.allclose(tables[7 * l + 3][1], ao, rtol=1e-6)
+        Wg, Wu = I.f16(m.weight(l, "gate")), I.f16(m.weight(l, "up"))
+        ad = I.silu_sq_moment((Wg * Wg) @ gm) * ((Wu * Wu) @ gm)
+        assert np.allclose(tables[7 * l + 6][1], ad, rtol=1e-6)
+        for j in (0, 1, 2, 4, 5):
+            assert tables[7 * l + j][2] is None
+        assert tables[7 * l + 3][2] is not None and tables[7 * l + 6][2] is not None
+    name, a_head, rho_head = tables[-1]
+    assert name == "lm_head" and rho_head is None
+    assert np.array_equal(a_head, sq_gain(m.gain(None, "final")).astype(np.float32))
+
+
 # ------------------------------------------------------- outlier rules
 
 @pytest.mark.parametrize("R", [7, 8])
