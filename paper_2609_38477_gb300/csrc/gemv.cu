@@ -53,7 +53,7 @@ struct Cfg {
   static constexpr int RW = (PIECES % 2) ? PIECES * 4 : PIECES * 4 + 4;
   static constexpr int STREAM_WORDS = 2 * 32 * RW;  // per warp, double-buffered
   static constexpr int XFLOATS = 2 * ST * 8 * NB;   // per warp, double-buffered
-  static constexpr int WARP_BYTES = STREAM_WORDS * 4 + XFLOATS * 4 + 2 * 32 * 8 * 2;
+  static constexpr int WARP_BYTES = STREAM_WORDS * 4 + XFLOATS * 4;
 };
 
 struct TensorArgs {
@@ -218,7 +218,7 @@ struct Piece {
 template <int NB>
 __device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t z,
                                            const uint64_t *tabs, uint32_t *sbuf, float *xbuf,
-                                           int16_t *bk, const Piece *pcs, int np, int nst_total,
+                                           const uint4 *rrec, const Piece *pcs, int np, int nst_total,
                                            float *comb, int warp, int lane) {
   using CF = Cfg<NB>;
   const LayerArgs &p = T.p;
@@ -226,6 +226,7 @@ __device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t 
   if (warp >= nst_total) return;
   const uint8_t *gstream = reinterpret_cast<const uint8_t *>(p.stream);
   int piece_of[2] = {0, 0}, cs_of[2] = {0, 0}, ce_of[2] = {0, 0};
+  int jr_of[2] = {0, 0}, nxt_of[2] = {0, 0};
   uint32_t pos0[2] = {0, 0};
 
   auto issue = [&](int t, int sb) {
@@ -237,27 +238,38 @@ __device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t 
       nsp = (pcs[pi].cb - pcs[pi].ca + CF::ST - 1) / CF::ST;
     }
     const int cs = pcs[pi].ca + t * CF::ST, ce = min(pcs[pi].cb, cs + CF::ST);
-    const int64_t r0 = pcs[pi].g * 32;
-    const int64_t ridx = r0 + lane;
-    const uint4 *rec = p.rowrec + 2 * (ridx < p.R ? ridx : r0);
-    const uint4 m0 = __ldg(rec), m1 = __ldg(rec + 1);
+    // The lane's row record (bit offset, breakpoints), staged for the round.
+    const uint4 m0 = rrec[(pi * 32 + lane) * 2], m1 = rrec[(pi * 32 + lane) * 2 + 1];
     const uint64_t roff = (uint64_t)m0.x | ((uint64_t)m0.y << 32);
-    int16_t *mybk = bk + (sb * 32 + lane) * 8;
-    *reinterpret_cast<uint4 *>(mybk) = make_uint4(m0.z, m0.w, m1.x, m1.y);
     const uint32_t bw[4] = {m0.z, m0.w, m1.x, m1.y};
     uint32_t s_cs, s_ce;
     lane_bits_before(bw, p, cs, ce, s_cs, s_ce);
+    // Rung of block cs (breakpoints at or below it) and the next breakpoint.
+    int jr0 = 0, nx0 = nb;
+#pragma unroll
+    for (int j = 0; j < kMaxJ - 1; ++j) {
+      const int b = (int)((bw[j >> 1] >> (16 * (j & 1))) & 0xffffu);
+      if (j < J - 1) {
+        jr0 += (b <= cs) ? 1 : 0;
+        if (b > cs) nx0 = min(nx0, b);
+      }
+    }
     const uint64_t bit_cs = roff + s_cs;
     const uint64_t b_lo = (bit_cs >> 3) & ~(uint64_t)15;
     uint64_t b_hi = (roff + s_ce + 96 + 7) >> 3;
     b_hi = (b_hi + 15) & ~(uint64_t)15;
-    if (b_hi > T.stream_bytes) b_hi = T.stream_bytes & ~(uint64_t)15;
+    if (b_hi > T.stream_bytes) {
+      // A stage reaching past the readable stream: the plan disagrees with
+      // the bound buffer.  Read only what is there and report it.
+      atomicOr(p.flags, 1u);
+      b_hi = T.stream_bytes & ~(uint64_t)15;
+    }
     const int npc = b_hi > b_lo ? (int)min((uint64_t)CF::PIECES, (b_hi - b_lo) >> 4) : 0;
     const uint32_t p0 = (uint32_t)(bit_cs - b_lo * 8);
     if (sb) {
-      piece_of[1] = pi; cs_of[1] = cs; ce_of[1] = ce; pos0[1] = p0;
+      piece_of[1] = pi; cs_of[1] = cs; ce_of[1] = ce; pos0[1] = p0; jr_of[1] = jr0; nxt_of[1] = nx0;
     } else {
-      piece_of[0] = pi; cs_of[0] = cs; ce_of[0] = ce; pos0[0] = p0;
+      piece_of[0] = pi; cs_of[0] = cs; ce_of[0] = ce; pos0[0] = p0; jr_of[0] = jr0; nxt_of[0] = nx0;
     }
     uint32_t *rows = sbuf + sb * 32 * CF::RW;
 #pragma unroll
@@ -299,12 +311,12 @@ __device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t 
       for (int b = 0; b < NB; ++b) acc[b] = 0.f;
       acc_piece = pi;
     }
-    const int16_t *mybk = bk + (sb * 32 + lane) * 8;
+    // The lane's breakpoints (int16, after the 8-byte bit offset of its record).
+    const int16_t *mybk = reinterpret_cast<const int16_t *>(rrec + (pi * 32 + lane) * 2) + 4;
     const uint32_t *rowbuf = sbuf + sb * 32 * CF::RW + lane * CF::RW;
     const float *xs = xbuf + sb * CF::ST * 8 * NB;
-    int jr = 0;
-    while (jr < J - 1 && mybk[jr] <= cs) ++jr;
-    int nxt = (jr < J - 1) ? mybk[jr] : nb;
+    int jr = sb ? jr_of[1] : jr_of[0];
+    int nxt = sb ? nxt_of[1] : nxt_of[0];
     // Passes over the stage's columns, each one run of blocks per lane at one
     // rung, all through a single call site (one inlined copy of the rung
     // loops keeps the instruction working set small).  Where all rows sit at
@@ -357,11 +369,11 @@ __device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t 
 }
 
 // Outlier epilogue: y_b[r] += sum_o W16[r, col_o] x_b[col_o] (Sec. 3.5).
-__device__ __forceinline__ float outlier_term(const TensorArgs &T, int64_t r, int b) {
+__device__ __forceinline__ float outlier_term(const LayerArgs &p, const uint16_t *x, int64_t r, int b) {
   float s = 0.f;
-  for (int o = 0; o < T.p.n_out; ++o) {
-    const float w = __half2float(__ushort_as_half(T.p.out_vals[r * T.p.n_out + o]));
-    s = __fmaf_rn(w, bf16_to_f32(T.x[(int64_t)b * T.p.C + T.p.out_cols[o]]), s);
+  for (int o = 0; o < p.n_out; ++o) {
+    const float w = __half2float(__ushort_as_half(p.out_vals[r * p.n_out + o]));
+    s = __fmaf_rn(w, bf16_to_f32(x[(int64_t)b * p.C + p.out_cols[o]]), s);
   }
   return s;
 }
@@ -380,9 +392,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ Mu
   uint8_t *mine = wbase + warp * CF::WARP_BYTES;
   uint32_t *sbuf = reinterpret_cast<uint32_t *>(mine);
   float *xbuf = reinterpret_cast<float *>(mine + CF::STREAM_WORDS * 4);
-  int16_t *bk = reinterpret_cast<int16_t *>(mine + CF::STREAM_WORDS * 4 + CF::XFLOATS * 4);
   float *comb = reinterpret_cast<float *>(wbase + kWarps * CF::WARP_BYTES);  // RG x kWarps x 32 x NB
-  int *flag = reinterpret_cast<int *>(comb + CF::RG * kWarps * 32 * NB);
+  uint4 *rrec = reinterpret_cast<uint4 *>(comb + CF::RG * kWarps * 32 * NB);  // RG x 32 x 2 row records
   {
     // The jump tables depend only on S, so any tensor's copy serves all.
     const uint4 *src = reinterpret_cast<const uint4 *>((kSet ? a.tens : a.t)[0].p.tables);
@@ -403,6 +414,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ Mu
   constexpr int kTWords = sizeof(TensorArgs) / 4;
   static_assert(sizeof(TensorArgs) % 8 == 0, "descriptor size");
   constexpr int kXWord = offsetof(TensorArgs, x) / 4, kYWord = offsetof(TensorArgs, y) / 4;
+  // Row groups cut by this CTA's range (at most two: where the range starts
+  // and where it ends inside a group): their partial sums go to slots during
+  // the rounds and are finished after the last round.  A: slot 0, B: slot 1.
+  int cutA_ti = -1, cutB_ti = -1, warpB = 0;
+  int64_t cutA_g = 0, cutB_g = 0;
+  int32_t crowA = -1, crowB = -1;
   int ti = 0;
   {
     int lo = 0, hi = a.nt - 1;  // last tensor whose first unit is <= u0
@@ -441,70 +458,126 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ Mu
     static_assert(CF::RG <= 8, "round size");
     int np = 0, nst_total = 0;
     int64_t uu = u;
+    const int ck = threadIdx.x >> 5, cln = threadIdx.x & 31;
+    int64_t cg = 0;
+    // Pieces whose row records this thread stages (record words i, i + kThreads).
+    const int rk0 = threadIdx.x >> 6, rk1 = (threadIdx.x + kThreads) >> 6;
+    int64_t rg0 = 0, rg1 = 0;
+    bool any_cut = false;  // the same in every thread
     while (uu < rend && np < CF::RG) {
       const int64_t lu = uu - tub;
       const int64_t g = lu / tnb;
       const int ca = (int)(lu - g * tnb);
       const int cbk = (int)min((int64_t)tnb, ca + (rend - uu));
       if (threadIdx.x == 0) pcs[np] = Piece{g, ca, cbk};
+      if (np == ck) cg = g;
+      if (np == rk0) rg0 = g;
+      if (np == rk1) rg1 = g;
+      any_cut |= !(ca == 0 && cbk == tnb);
       nst_total += (cbk - ca + CF::ST - 1) / CF::ST;
       ++np;
       uu += cbk - ca;
     }
+    // The output rows of the round, loaded now (thread t < 32 np: row t % 32
+    // of piece t / 32): the loads complete during the round; volatile keeps
+    // them ahead of the round's copies.
+    __shared__ int32_t srow[8 * 32];
+    int32_t crow = -1;
+    if (ck < np && cg * 32 + cln < p.R) {
+      const int32_t *ap = p.rowperm + cg * 32 + cln;
+      asm volatile("{\n\t.reg .u64 ga;\n\tcvta.to.global.u64 ga, %1;\n\tld.global.nc.b32 %0, [ga];\n\t}"
+                   : "=r"(crow) : "l"(ap));
+    }
     for (int i = threadIdx.x; i < np * kWarps * 32 * NB; i += kThreads) comb[i] = 0.f;
-    __syncthreads();
-    warp_round<NB>(T, a.n, a.zero, tabs, sbuf, xbuf, bk, pcs, np, nst_total, comb, warp, lane);
-    __syncthreads();
-    for (int k = 0; k < np; ++k) {
-      const int64_t g = pcs[k].g, r0 = g * 32;
-      const bool full = (pcs[k].ca == 0 && pcs[k].cb == p.nb);
-      const int sidx = (k == 0 && first) ? 0 : 1;
-      for (int i = threadIdx.x; i < 32 * NB; i += kThreads) {
-        float v = 0.f;
-        for (int w = 0; w < kWarps; ++w) v += comb[(k * kWarps + w) * 32 * NB + i];
-        const int ln = i / NB, b = i - ln * NB;
-        if (full) {
-          if (r0 + ln < p.R && b < a.n) {
-            const int64_t rr = __ldg(p.rowperm + r0 + ln);
-            T.y[(int64_t)b * p.R + rr] = v + outlier_term(T, rr, b);
-          }
-        } else {
-          p.slots[((int64_t)cta * 2 + sidx) * 32 * kMaxBatch + i] = v;
-        }
+    // The round's row records (32 bytes per row of each piece; rows past R
+    // repeat the group's first row), read once per round.
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int i = threadIdx.x + h * kThreads;
+      const int k = h ? rk1 : rk0;
+      if (k < np) {
+        const int64_t r0 = (h ? rg1 : rg0) * 32, ridx = r0 + ((i >> 1) & 31);
+        rrec[i] = __ldg(tens[ti].p.rowrec + 2 * (ridx < tens[ti].p.R ? ridx : r0) + (i & 1));
       }
-      if (!full) {
-        const int64_t gu = T.ubegin + g * p.nb;
-        __syncthreads();
-        if (threadIdx.x == 0) {
-          __threadfence();
-          const int cf = cta_of(cb, a.ctas, gu), cl = cta_of(cb, a.ctas, gu + p.nb - 1);
-          const int old = atomicAdd(p.counters + g, 1);
-          *flag = (old == cl - cf) ? 1 : 0;
-        }
-        __syncthreads();
-        if (*flag) {
-          __threadfence();
-          const int cf = cta_of(cb, a.ctas, gu), cl = cta_of(cb, a.ctas, gu + p.nb - 1);
-          for (int i = threadIdx.x; i < 32 * NB; i += kThreads) {
-            float v = 0.f;
-            for (int c2 = cf; c2 <= cl; ++c2) {
-              const int s2 = (cb[c2] >= gu) ? 0 : 1;
-              v += __ldcg(p.slots + ((int64_t)c2 * 2 + s2) * 32 * kMaxBatch + i);
-            }
-            const int ln = i / NB, b = i - ln * NB;
-            if (r0 + ln < p.R && b < a.n) {
-              const int64_t rr = __ldg(p.rowperm + r0 + ln);
-              T.y[(int64_t)b * p.R + rr] = v + outlier_term(T, rr, b);
-            }
-          }
-          if (threadIdx.x == 0) p.counters[g] = 0;
-        }
-        __syncthreads();
+    }
+    __syncthreads();
+    warp_round<NB>(T, a.n, a.zero, tabs, sbuf, xbuf, rrec, pcs, np, nst_total, comb, warp, lane);
+    if (ck < np) srow[threadIdx.x] = crow;
+    __syncthreads();
+    // Row sums of the round's pieces (warps added in warp order), every (piece,
+    // row, batch column) at once: full row groups go to y, cut ones to this
+    // CTA's partial-sum slot (slot 0: the first piece of the CTA's range,
+    // slot 1: its last piece).
+    for (int i = threadIdx.x; i < np * 32 * NB; i += kThreads) {
+      const int k = i / (32 * NB), rem = i - k * 32 * NB, b = rem % NB;
+      float v = 0.f;
+      for (int w = 0; w < kWarps; ++w) v += comb[(k * kWarps + w) * 32 * NB + rem];
+      if (pcs[k].ca == 0 && pcs[k].cb == p.nb) {
+        const int32_t rr = srow[k * 32 + rem / NB];
+        if (rr >= 0 && b < a.n) T.y[(int64_t)b * p.R + rr] = v + outlier_term(p, T.x, rr, b);
+      } else {
+        const int sidx = (k == 0 && first) ? 0 : 1;
+        p.slots[((int64_t)cta * 2 + sidx) * 32 * kMaxBatch + rem] = v;
+      }
+    }
+    if (any_cut) {
+      const bool c0 = first && !(pcs[0].ca == 0 && pcs[0].cb == p.nb);
+      const bool cl = !(pcs[np - 1].ca == 0 && pcs[np - 1].cb == p.nb) && !(first && np == 1);
+      if (c0) {
+        cutA_ti = ti;
+        cutA_g = pcs[0].g;
+        if (ck == 0) crowA = crow;
+      }
+      if (cl) {
+        cutB_ti = ti;
+        cutB_g = pcs[np - 1].g;
+        warpB = np - 1;
+        if (ck == np - 1) crowB = crow;
       }
     }
     __syncthreads();
     first = false;
     u = uu;
+  }
+  if (cutA_ti >= 0 || cutB_ti >= 0) {
+    // Each CTA publishes its partial sums of a cut row group and counts its
+    // arrival; the CTA that arrives last adds the slots in CTA order and
+    // writes y.  No CTA waits for another.  (The last round ended with a
+    // barrier, so this CTA's slot writes precede the fence.)
+    __shared__ int sflag[2];
+    const int side = threadIdx.x == 0 ? 0 : threadIdx.x == 32 ? 1 : -1;
+    if (side >= 0 && (side ? cutB_ti : cutA_ti) >= 0) {
+      const TensorArgs &TX = tens[side ? cutB_ti : cutA_ti];
+      const int64_t g = side ? cutB_g : cutA_g, gu = TX.ubegin + g * TX.p.nb;
+      const int cf = cta_of(cb, a.ctas, gu), cl = cta_of(cb, a.ctas, gu + TX.p.nb - 1);
+      __threadfence();
+      const int old = atomicAdd(TX.p.counters + g, 1);
+      const bool last = (old == cl - cf);
+      if (last) __threadfence();
+      sflag[side] = last ? 1 : 0;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int side = 0; side < 2; ++side) {
+      const int xti = side ? cutB_ti : cutA_ti;
+      if (xti < 0 || warp != (side ? warpB : 0) || !sflag[side]) continue;
+      const TensorArgs &TX = tens[xti];
+      const int64_t g = side ? cutB_g : cutA_g, gu = TX.ubegin + g * TX.p.nb;
+      const int cf = cta_of(cb, a.ctas, gu), cl = cta_of(cb, a.ctas, gu + TX.p.nb - 1);
+      const int32_t rr = side ? crowB : crowA;
+      float *y = kSet ? a.Yall + (int64_t)a.n * TX.rpre : TX.y;
+      const uint16_t *x = kSet ? a.Xall + (int64_t)a.n * TX.cpre : TX.x;
+#pragma unroll
+      for (int b = 0; b < NB; ++b) {
+        float v = 0.f;
+        for (int c2 = cf; c2 <= cl; ++c2) {
+          const int s2 = (cb[c2] >= gu) ? 0 : 1;
+          v += __ldcg(TX.p.slots + ((int64_t)c2 * 2 + s2) * 32 * kMaxBatch + lane * NB + b);
+        }
+        if (rr >= 0 && b < a.n) y[(int64_t)b * TX.p.R + rr] = v + outlier_term(TX.p, x, rr, b);
+      }
+      if (lane == 0) TX.p.counters[g] = 0;
+    }
   }
 }
 
@@ -571,7 +644,7 @@ __global__ void k_xperm_set(const TensorArgs *__restrict__ tens, const uint16_t 
 template <int NB>
 static size_t smem_bytes() {
   return sizeof(uint64_t) * 512 * kTableSlots + (size_t)kWarps * Cfg<NB>::WARP_BYTES +
-         sizeof(float) * Cfg<NB>::RG * kWarps * 32 * NB + 16;
+         sizeof(float) * Cfg<NB>::RG * kWarps * 32 * NB + sizeof(uint4) * Cfg<NB>::RG * 32 * 2;
 }
 
 // Cost-balanced ranges of the units of all tensors, one per CTA.  A group's
