@@ -334,7 +334,7 @@ seedq_status seedq_synth_stream(const seedq_layer *layer, uint64_t key,
  * cudaMalloc when they need it (a fixed memory budget reserved up front, an
  * allocator-less runtime, code that must not touch the CUDA allocator while
  * other work is in flight).  The paper has no counterpart: it is the row part
- * of seedq_layer_prepare (Eq. ladder breakpoints, the tie pass, row bit
+ * of seedq_layer_prepare (per-row rung breakpoints, the tie pass, row bit
  * offsets) run on caller buffers, with its temporary per-row tie counts in a
  * file-scope device array of SEEDQ_STATIC_PLAN_MAX_ROWS entries (512 KiB held
  * by every GPU that loads the library until exit).  It allocates nothing.
@@ -347,8 +347,10 @@ seedq_status seedq_synth_stream(const seedq_layer *layer, uint64_t key,
  *   row_off   device, rows + 1 uint64 out (row_off[rows] = total bits).
  *   summary   device, 2 uint64 out: tied blocks at theta[j_tie], total bits;
  *             the caller checks tie_count <= summary[0].
- * The first call on a device looks up the array's device address with that
- * device current, so make it before any stream capture.  Work is enqueued on
+ * Every call looks up the array's device address with the current device; the
+ * first call on a device also loads the library's module there, so make it
+ * before any stream capture.  The rung lengths travel in the kernel
+ * parameters, so the call makes no host-to-device copy.  Work is enqueued on
  * cuda_stream and not waited for.  Calls share the array: calls that overlap
  * on the GPU (other streams, other threads) race and must be serialized. */
 #define SEEDQ_STATIC_PLAN_MAX_ROWS (1 << 17)

@@ -2,6 +2,7 @@
 from __future__ import annotations
 
 import concurrent.futures as cf
+import glob
 import os
 import subprocess
 
@@ -11,7 +12,9 @@ CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libseedq.so")
 SOURCES = ["plan.cu", "decode.cu", "gemv.cu", "encode.cu", "importance.cu", "container.cpp"]
-HEADERS = [os.path.join(CSRC, "seedq_internal.cuh"), os.path.join(ROOT, "include", "seedq.h")]
+# Every header a translation unit may include: an edit to any of them rebuilds all objects.
+HEADERS = sorted(glob.glob(os.path.join(CSRC, "*.cuh")) + glob.glob(os.path.join(CSRC, "*.h")) +
+                 glob.glob(os.path.join(ROOT, "include", "*.h")))
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC"] + ARCH
 

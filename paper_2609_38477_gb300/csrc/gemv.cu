@@ -28,6 +28,7 @@
 #include <vector>
 
 #include "cp_async.cuh"
+#include "device_once.h"
 #include "f32x2.cuh"
 #include "seedq_internal.cuh"
 
@@ -218,7 +219,8 @@ struct Piece {
 template <int NB>
 __device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t z,
                                            const uint64_t *tabs, uint32_t *sbuf, float *xbuf,
-                                           const uint4 *rrec, const Piece *pcs, int np, int nst_total,
+                                           const uint4 *rrec, const Piece *pcs, const int *pst, int np,
+                                           int nst_total,
                                            float *comb, int warp, int lane) {
   using CF = Cfg<NB>;
   const LayerArgs &p = T.p;
@@ -230,14 +232,12 @@ __device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t 
   uint32_t pos0[2] = {0, 0};
 
   auto issue = [&](int t, int sb) {
+    // Piece of stage t: the number of pieces after the first whose first
+    // stage is at or before t (independent loads, no dependent chain).
     int pi = 0;
-    int nsp = (pcs[0].cb - pcs[0].ca + CF::ST - 1) / CF::ST;
-    while (t >= nsp && pi + 1 < np) {
-      t -= nsp;
-      ++pi;
-      nsp = (pcs[pi].cb - pcs[pi].ca + CF::ST - 1) / CF::ST;
-    }
-    const int cs = pcs[pi].ca + t * CF::ST, ce = min(pcs[pi].cb, cs + CF::ST);
+#pragma unroll
+    for (int k = 1; k < CF::RG; ++k) pi += (k < np && t >= pst[k]) ? 1 : 0;
+    const int cs = pcs[pi].ca + (t - pst[pi]) * CF::ST, ce = min(pcs[pi].cb, cs + CF::ST);
     // The lane's row record (bit offset, breakpoints), staged for the round.
     const uint4 m0 = rrec[(pi * 32 + lane) * 2], m1 = rrec[(pi * 32 + lane) * 2 + 1];
     const uint64_t roff = (uint64_t)m0.x | ((uint64_t)m0.y << 32);
@@ -455,6 +455,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ Mu
     // The next round: up to RG row groups of this tensor.
     // (In shared memory: the stage issue indexes it by a runtime piece number.)
     __shared__ Piece pcs[8];
+    __shared__ int pst[8];  // first stage of each piece in the round's stage order
     static_assert(CF::RG <= 8, "round size");
     int np = 0, nst_total = 0;
     int64_t uu = u;
@@ -469,7 +470,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ Mu
       const int64_t g = lu / tnb;
       const int ca = (int)(lu - g * tnb);
       const int cbk = (int)min((int64_t)tnb, ca + (rend - uu));
-      if (threadIdx.x == 0) pcs[np] = Piece{g, ca, cbk};
+      if (threadIdx.x == 0) {
+        pcs[np] = Piece{g, ca, cbk};
+        pst[np] = nst_total;
+      }
       if (np == ck) cg = g;
       if (np == rk0) rg0 = g;
       if (np == rk1) rg1 = g;
@@ -501,7 +505,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ Mu
       }
     }
     __syncthreads();
-    warp_round<NB>(T, a.n, a.zero, tabs, sbuf, xbuf, rrec, pcs, np, nst_total, comb, warp, lane);
+    warp_round<NB>(T, a.n, a.zero, tabs, sbuf, xbuf, rrec, pcs, pst, np, nst_total, comb, warp, lane);
     if (ck < np) srow[threadIdx.x] = crow;
     __syncthreads();
     // Row sums of the round's pieces (warps added in warp order), every (piece,
@@ -647,6 +651,38 @@ static size_t smem_bytes() {
          sizeof(float) * Cfg<NB>::RG * kWarps * 32 * NB + sizeof(uint4) * Cfg<NB>::RG * 32 * 2;
 }
 
+// The fused kernel's dynamic shared-memory limit is a per-device attribute:
+// set once per device (any host thread), and set again if a launch reports an
+// invalid configuration (the device's context may have been reset since).
+template <int NB, bool kSet>
+static DeviceOnce &smem_once() {
+  static DeviceOnce once;
+  return once;
+}
+
+template <int NB, bool kSet>
+static cudaError_t set_smem_limit(int dev) {
+  return (cudaError_t)smem_once<NB, kSet>().run(dev, [] {
+    return (int)cudaFuncSetAttribute(k_gemv<NB, kSet>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)smem_bytes<NB>());
+  });
+}
+
+template <int NB, bool kSet>
+static cudaError_t launch_fused(const cudaLaunchConfig_t &cfg, const MultiArgs &a) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = set_smem_limit<NB, kSet>(dev);
+  if (e == cudaSuccess) e = cudaLaunchKernelEx(&cfg, k_gemv<NB, kSet>, a);
+  if (e == cudaErrorInvalidValue) {
+    (void)cudaGetLastError();
+    smem_once<NB, kSet>().forget(dev);
+    e = set_smem_limit<NB, kSet>(dev);
+    if (e == cudaSuccess) e = cudaLaunchKernelEx(&cfg, k_gemv<NB, kSet>, a);
+  }
+  return e;
+}
+
 // Cost-balanced ranges of the units of all tensors, one per CTA.  A group's
 // cost is its modeled time at batch n (block passes and the sum of k over
 // them); inside the group where a range is cut, the first row's rung profile,
@@ -745,15 +781,8 @@ static seedq_status launch(const seedq_layer *const *layers, int nt, const uint1
   a->cbd = nullptr;
   a->Xall = nullptr;
   a->Yall = nullptr;
-  static bool attr_set = false;
   seedq_status rc = SEEDQ_OK;
-  if (!attr_set) {
-    const cudaError_t e = cudaFuncSetAttribute(k_gemv<NB, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               (int)smem_bytes<NB>());
-    if (e != cudaSuccess) rc = cuda_fail(e);
-    else attr_set = true;
-  }
-  if (rc == SEEDQ_OK) {
+  {
     XpermArgs xa;
     xa.n = n;
     xa.nbt = NB;
@@ -786,7 +815,7 @@ static seedq_status launch(const seedq_layer *const *layers, int nt, const uint1
       attr[0].val.programmaticStreamSerializationAllowed = 1;
       cfg.attrs = attr;
       cfg.numAttrs = 1;
-      e = cudaLaunchKernelEx(&cfg, k_gemv<NB, false>, *a);
+      e = launch_fused<NB, false>(cfg, *a);
     }
     if (e != cudaSuccess) rc = cuda_fail(e);
   }
@@ -833,13 +862,6 @@ static int tmpl_index(int nb) { return nb <= 1 ? 0 : nb <= 2 ? 1 : nb <= 4 ? 2 :
 template <int NB>
 static seedq_status launch_set(const seedq_layer_set *S, const uint16_t *X, int n, float *Y,
                                cudaStream_t st) {
-  static bool attr_set = false;
-  if (!attr_set) {
-    const cudaError_t e = cudaFuncSetAttribute(k_gemv<NB, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               (int)smem_bytes<NB>());
-    if (e != cudaSuccess) return cuda_fail(e);
-    attr_set = true;
-  }
   MultiArgs a;
   memset(&a, 0, sizeof a);
   a.nt = S->nt;
@@ -865,7 +887,7 @@ static seedq_status launch_set(const seedq_layer_set *S, const uint16_t *X, int 
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, k_gemv<NB, true>, a);
+    e = launch_fused<NB, true>(cfg, a);
   }
   return e == cudaSuccess ? SEEDQ_OK : cuda_fail(e);
 }

@@ -258,12 +258,17 @@ __device__ uint64_t block_exclusive_scan(uint64_t v, uint64_t *sh, uint64_t *tot
 // Tie pass of Alg. 2 (the first T tied blocks in row-major order take the lower
 // rung) applied to the breakpoints, then per-row bit counts and their exclusive
 // scan into row offsets.  One CTA of 1024 threads, rows in contiguous chunks.
-__global__ void k_scan(int64_t R, int J, int nb, int j_tie, int64_t T, const int *Lrung,
+// Block bits of each rung, passed by value in the kernel's parameters.
+struct RungBits {
+  int32_t L[kMaxJ];
+};
+
+__global__ void k_scan(int64_t R, int J, int nb, int j_tie, int64_t T, const RungBits Lrung,
                        int32_t *__restrict__ brk, const int32_t *__restrict__ tcnt,
                        uint64_t *__restrict__ row_off, uint64_t *__restrict__ summary) {
   __shared__ uint64_t sh[1024];
   __shared__ int L[kMaxJ];
-  if (threadIdx.x < J) L[threadIdx.x] = Lrung[threadIdx.x];
+  if (threadIdx.x < J) L[threadIdx.x] = Lrung.L[threadIdx.x];
   const int64_t per = (R + blockDim.x - 1) / blockDim.x;
   const int64_t r0 = min((int64_t)threadIdx.x * per, R), r1 = min(r0 + per, R);
   uint64_t tied_total = 0;
@@ -628,10 +633,9 @@ seedq_status seedq_layer_prepare(const seedq_layer_desc *d, const seedq_schedule
 
   L->args.stream = nullptr;
 
-  int *dL = nullptr;
-  cudaError_t e = cudaMalloc((void **)&dL, sizeof(int) * kMaxJ);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(dL, L->args.L, sizeof(int) * kMaxJ, cudaMemcpyHostToDevice, st);
-  if (e == cudaSuccess) e = cudaMemsetAsync(L->d_flags, 0, sizeof(uint32_t), st);
+  RungBits rb;
+  for (int j = 0; j < kMaxJ; ++j) rb.L[j] = L->args.L[j];
+  cudaError_t e = cudaMemsetAsync(L->d_flags, 0, sizeof(uint32_t), st);
   if (e == cudaSuccess) e = cudaMemcpyAsync(L->d_a_in, d->a, sizeof(float) * C, cudaMemcpyHostToDevice, st);
   if (e == cudaSuccess && d->rho)
     e = cudaMemcpyAsync(L->d_rho_in, d->rho, sizeof(float) * R, cudaMemcpyHostToDevice, st);
@@ -651,7 +655,7 @@ seedq_status seedq_layer_prepare(const seedq_layer_desc *d, const seedq_schedule
     } else {
       e = cudaMemsetAsync(L->d_tcnt, 0, sizeof(int32_t) * R, st);
     }
-    k_scan<<<1, 1024, 0, st>>>(R, J, nb, J > 1 ? s->j_tie : -1, d->tie_count, dL, L->d_brk,
+    k_scan<<<1, 1024, 0, st>>>(R, J, nb, J > 1 ? s->j_tie : -1, d->tie_count, rb, L->d_brk,
                                L->d_tcnt, L->d_row_off, L->d_summary);
     bool rho_uniform = true;
     if (d->rho)
@@ -669,7 +673,6 @@ seedq_status seedq_layer_prepare(const seedq_layer_desc *d, const seedq_schedule
   uint64_t summary[2] = {0, 0};
   if (e == cudaSuccess) e = cudaMemcpyAsync(summary, L->d_summary, sizeof summary, cudaMemcpyDeviceToHost, st);
   if (e == cudaSuccess) e = cudaStreamSynchronize(st);
-  cudaFree(dL);
   if (e != cudaSuccess) {
     free_layer(L);
     return cuda_fail(e);
@@ -804,32 +807,23 @@ constexpr int64_t kStaticPlanMaxRows = 1 << 17;
 
 struct StaticPlanScratch {
   int32_t tcnt[kStaticPlanMaxRows];
-  int32_t L[kMaxJ];
 };
 
 static __device__ __align__(256) StaticPlanScratch g_static_plan_scratch;
 
-// Device address of the array, looked up once per device with that device
-// current (in host code the symbol is only a host-side stand-in).
+// Device address of the array on the current device (in host code the symbol
+// is only a host-side stand-in).  Looked up on every call: the first lookup on
+// a device loads the module there, later ones are cheap, and an address is
+// never reused from a context that has since been destroyed.
 static StaticPlanScratch *static_scratch_ptr(seedq_status *st) {
-  static StaticPlanScratch *ptrs[64] = {nullptr};
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess || dev < 0 || dev >= 64) {
-    *st = e != cudaSuccess ? cuda_fail(e) : SEEDQ_ERR_UNSUPPORTED;
+  void *p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_static_plan_scratch);
+  if (e != cudaSuccess) {
+    *st = cuda_fail(e);
     return nullptr;
   }
-  if (!ptrs[dev]) {
-    void *p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_static_plan_scratch);
-    if (e != cudaSuccess) {
-      *st = cuda_fail(e);
-      return nullptr;
-    }
-    ptrs[dev] = (StaticPlanScratch *)p;
-  }
   *st = SEEDQ_OK;
-  return ptrs[dev];
+  return (StaticPlanScratch *)p;
 }
 
 }  // namespace seedq
@@ -858,9 +852,8 @@ extern "C" seedq_status seedq_row_plan_static(const double *abar, const double *
   StaticPlanScratch *scr = static_scratch_ptr(&st);
   if (!scr) return st;
   cudaStream_t cs = (cudaStream_t)cuda_stream;
-  int32_t L[kMaxJ] = {0};
-  for (int j = 0; j < s->J; ++j) L[j] = s->rungs[j].S + 4 * s->rungs[j].k + 4;
-  SEEDQ_CUDA(cudaMemcpyAsync(scr->L, L, sizeof L, cudaMemcpyHostToDevice, cs));
+  RungBits rb;
+  for (int j = 0; j < kMaxJ; ++j) rb.L[j] = j < s->J ? s->rungs[j].S + 4 * s->rungs[j].k + 4 : 0;
   SchedArgs sa;
   sa.J = s->J;
   sa.j_tie = s->j_tie;
@@ -870,7 +863,7 @@ extern "C" seedq_status seedq_row_plan_static(const double *abar, const double *
   // array needs no clearing; with a single rung there are no ties to count.
   if (s->J > 1)
     k_rows<<<(int)((rows + 255) / 256), 256, 0, cs>>>(abar, rho, nb, rows, sa, brk, scr->tcnt);
-  k_scan<<<1, 1024, 0, cs>>>(rows, s->J, nb, s->J > 1 ? s->j_tie : -1, tie_count, scr->L, brk,
+  k_scan<<<1, 1024, 0, cs>>>(rows, s->J, nb, s->J > 1 ? s->j_tie : -1, tie_count, rb, brk,
                              scr->tcnt, row_off, summary);
   SEEDQ_CUDA(cudaGetLastError());
   return SEEDQ_OK;

@@ -557,39 +557,119 @@ def test_encoder_beats_other_seeds_lstsq():
 
 def test_round_trip_64x64_mixed_rungs():
     """Encode a 64x64 matrix with the oracle's seed search at the rungs the
-    schedule assigns (S <= 12 hull, plus one row forced through S = 16), pack,
-    decode: the decoder reproduces the encoder's reconstruction bit for bit."""
+    schedule assigns (four rungs, the last block column of every row at S = 16),
+    pack, decode: the decoder reproduces the encoder's reconstruction bit for bit
+    (Sec. 3.1 seed search, Alg. 2 decode)."""
     rng = np.random.default_rng(11)
     R = Cc = 64
     a = np.exp(rng.normal(0, 1, Cc)).astype(np.float32)
     t = O.Tensor(R, Cc, a)
+    ab = t.abar
+    assert ab[7] > ab[6]
     rungs = [(8, 3), (10, 3), (12, 3), (16, 3)]
-    s = O.Sched(rungs, [0.6, 1.0, 1e300], -1, 0.0)  # (16,3) never by threshold
+    # thresholds below the top block mean, the last one between the two largest
+    th = [float(ab[2]), float(ab[5]), float((ab[6] + ab[7]) / 2)]
+    s = O.Sched(rungs, th, -1, 0.0)
     rm = t.rung_rows(s, 0)
-    assert len(set(rm.ravel().tolist())) >= 2
+    assert set(rm.ravel().tolist()) == {0, 1, 2, 3}
+    assert np.all(rm[:, 7] == 3) and np.all(rm[:, :7] < 3)
     Wt = rng.normal(0, 0.02, (R, Cc))
     stream = np.zeros(64 * 8 * 6 + 64, np.uint8)
     ref = np.zeros((R, Cc), np.float32)
+    errs = np.zeros((R, Cc // 8))
     pos = 0
     for r in range(R):
         for c in range(Cc // 8):
             S, k = rungs[rm[r, c]]
-            if r == 63 and c < 2:  # S = 16 blocks are not reachable by this schedule
-                pass
             blk = Wt[r, t.perm[8 * c:8 * c + 8]]
-            seed, E, tt, _ = O.encode_block(S, k, O.find_taps(S), blk)
+            seed, E, tt, err = O.encode_block(S, k, O.find_taps(S), blk)
             O.write_bits(stream, pos, S, seed)
             O.write_bits(stream, pos + S, 4, E & 15)
             for j in range(k):
                 O.write_bits(stream, pos + S + 4 + 4 * j, 4, tt[j] & 15)
             pos += O.block_bits(S, k)
-            ref[r, t.perm[8 * c:8 * c + 8]] = O.reconstruct_block(S, k, O.find_taps(S), seed, E, tt)
+            rec = O.reconstruct_block(S, k, O.find_taps(S), seed, E, tt)
+            ref[r, t.perm[8 * c:8 * c + 8]] = rec
+            errs[r, c] = err
+            assert abs(float(((blk - rec.astype(np.float64)) ** 2).sum()) - err) <= 1e-15
+    assert pos == t.row_bit_offset(s, 0, R)
     dec = t.decode_rows(s, 0, stream, pos)
     assert np.array_equal(dec, ref)
-    # S = 16: one row of blocks encoded and reconstructed through the same path.
-    taps16 = O.find_taps(16)
-    for c in range(2):
-        blk = Wt[0, 8 * c:8 * c + 8]
-        seed, E, tt, err = O.encode_block(16, 3, taps16, blk)
-        rec = O.reconstruct_block(16, 3, taps16, seed, E, tt).astype(np.float64)
-        assert abs(float(((blk - rec) ** 2).sum()) - err) <= 1e-15
+    # A wider seed space fits at least as well on average (more seeds searched).
+    assert errs[:, 7].mean() < errs[:, 0].mean()
+
+
+# ------------------------------------------- checker helpers of the GPU tests
+#
+# or_synth_gemv_threads (the fp64 y reference of the large parity tests),
+# or_synth_pack_rows (the reference of the device stream bits) and
+# or_decode_gemv_threads, pinned to a whole-tensor left-to-right parse
+# (Alg. 2 with the tie counter running from row 0) on a tensor whose tied group
+# spans every row and is only partly demoted, so a row range starting inside
+# the demoted part needs the right carry-in.
+
+def _tie_case():
+    rng = np.random.default_rng(21)
+    R, Cc = 64, 256
+    a = np.exp(rng.normal(0, 0.7, Cc)).astype(np.float32)
+    t = O.Tensor(R, Cc, a)
+    ab = t.abar
+    assert len(set(ab.tolist())) == Cc // 8
+    cstar = 20
+    # thresholds: one between block means, one exactly at block column cstar's
+    # mean, whose tied group (column cstar of every row, rho = 1) is demoted
+    # for its first T members only
+    s = O.Sched([(8, 3), (12, 3), (16, 3)], [float(ab[10]), float(ab[cstar])], 1, 0.0)
+    T = 20
+    assert t.tied_blocks(s) == R
+    full_rm = t.rung_rows(s, T)
+    assert np.all(full_rm[:T, cstar] == 1) and np.all(full_rm[T:, cstar] == 2)
+    key = 0x5EED
+    stream, bits = t.synth_pack(s, T, key)
+    full = t.decode_rows(s, T, stream, bits)
+    L = np.array([O.block_bits(S, k) for S, k in s.rungs], np.int64)
+    off = np.concatenate([[0], np.cumsum(L[full_rm].sum(axis=1))])
+    assert off[-1] == bits
+    return t, s, T, key, stream, bits, full, off
+
+
+def _exact_y(Wm, x, nb):
+    import math
+    xf = W.bf16_bits_to_f32(x).astype(np.float64).reshape(nb, -1)
+    Wd = Wm.astype(np.float64)
+    y = np.array([[math.fsum(Wd[r] * xf[b]) for r in range(Wd.shape[0])] for b in range(nb)])
+    ya = np.abs(xf) @ np.abs(Wd).T
+    return y, ya
+
+
+@pytest.mark.parametrize("nb", [1, 3, 16])
+@pytest.mark.parametrize("r0,n", [(0, 64), (15, 10), (20, 9), (37, 27)])
+def test_synth_gemv_threads_pinned(nb, r0, n):
+    t, s, T, key, stream, bits, full, off = _tie_case()
+    rng = np.random.default_rng(nb * 100 + r0)
+    x = W.to_bf16_bits(rng.normal(0, 1, nb * t.C).astype(np.float32)).reshape(nb, t.C)
+    y, ya = t.synth_gemv(s, T, key, x, r0, n, nthreads=3)
+    ry, rya = _exact_y(full[r0:r0 + n], x, nb)
+    assert y.shape == (nb, n)
+    assert np.all(np.abs(y - ry) <= 1e-13 * rya + 1e-300)
+    assert np.allclose(ya, rya, rtol=1e-13, atol=0)
+    # the rows themselves, generated from the same carry-in
+    assert np.array_equal(t.synth_rows(s, T, key, r0, n), full[r0:r0 + n])
+
+
+@pytest.mark.parametrize("r0,n", [(0, 5), (15, 10), (19, 2), (20, 44)])
+def test_synth_pack_rows_is_a_slice(r0, n):
+    t, s, T, key, stream, bits, full, off = _tie_case()
+    part, pbits = t.synth_pack_rows(s, T, key, r0, n, int(off[r0 + n] - off[r0]))
+    assert pbits == off[r0 + n] - off[r0]
+    allbits = np.unpackbits(stream, bitorder="little")[off[r0]:off[r0 + n]]
+    assert np.array_equal(np.unpackbits(part, bitorder="little")[:pbits], allbits)
+
+
+@pytest.mark.parametrize("r0,n", [(15, 10), (33, 31)])
+def test_decode_gemv_threads_row_range(r0, n):
+    t, s, T, key, stream, bits, full, off = _tie_case()
+    x = W.x_bf16(W.WORKLOADS["c0"], 0, 2)[:, :t.C].copy()
+    y, used = t.decode_gemv_threads(s, T, stream, bits, x, 4, r0, n)
+    ry, rya = _exact_y(full[r0:r0 + n], x, 2)
+    assert np.all(np.abs(y[:, r0:r0 + n] - ry) <= 1e-13 * rya + 1e-300)
