@@ -129,6 +129,16 @@ uint64_t seedq_stream_bytes_required(uint64_t bits);
 seedq_status seedq_layer_bind_stream(seedq_layer *layer, const void *stream,
                                      uint64_t stream_bits, uint64_t stream_bytes);
 
+/* Diagnostics: lower the number of bound-stream bytes the layer's kernels may
+ * read to `bytes` (at most the bound size; it cannot be raised again without
+ * binding anew).  With fewer bytes than seedq_stream_bytes_required(bits) the
+ * kernels cut their reads off at the limit and set bit 0 of the device error
+ * flags; the results are then wrong for the rows that reach the limit.  Used to
+ * test the error flag without any out-of-bounds access.  No paper counterpart.
+ * Errors: INVALID_ARG (NULL layer, bytes above the bound size), STREAM
+ * (unbound). */
+seedq_status seedq_layer_limit_stream_bytes(seedq_layer *layer, uint64_t bytes);
+
 /* Free the plan (waits for the device).  NULL is accepted. */
 seedq_status seedq_layer_release(seedq_layer *layer);
 
@@ -223,9 +233,13 @@ seedq_status seedq_layer_perm(const seedq_layer *layer, int32_t *perm_host);
  * Synchronous.  Errors: INVALID_ARG (NULL pointer), CUDA. */
 seedq_status seedq_layer_row_offsets(const seedq_layer *layer, uint64_t *offsets_host);
 
-/* Device error flags accumulated by the layer's kernels since prepare (bit 0:
- * a block offset disagreed with the row offsets; bit 1: unbound stream).
- * Synchronous; 0 means no fault was seen. */
+/* Device error flags accumulated by the layer's kernels since prepare.  Bit 0:
+ * the plan and the bound buffer disagree -- a kernel's read range reached past
+ * the readable bytes of the stream (the read is cut off there, the affected
+ * weights or rows are wrong, nothing outside the buffer is read), or the bits a
+ * row's blocks occupy by its rung breakpoints differ from its row offsets.
+ * Never set for a stream bound with seedq_layer_bind_stream and a plan from
+ * seedq_layer_prepare.  Synchronous; 0 means no fault was seen. */
 seedq_status seedq_last_device_error(const seedq_layer *layer, uint32_t *flags);
 
 /* Tap mask T_S of the width-S LFSR used by the stream format (bit i set when
@@ -272,6 +286,17 @@ seedq_status seedq_encode_layer(const seedq_layer *layer, const float *W, uint32
 seedq_status seedq_pack_stream(const seedq_layer *layer, const uint32_t *seed, const int8_t *E,
                                const int8_t *t, void *stream, uint64_t stream_bytes,
                                void *cuda_stream);
+
+/* Measurement helper for the encoder's roofline (no paper counterpart): one
+ * launch of blocks_per_sm x SMs CTAs of 256 threads, each thread running eight
+ * independent fp64 FMA chains for `iters` steps, so the device's fp64 FMA
+ * pipe bounds it.  *fmas receives the FMAs the launch performs (2 flops each);
+ * the caller times it on cuda_stream.  out: device, one double (written only
+ * in a case that does not arise; it keeps the chains from being removed).
+ * Asynchronous.  Errors: INVALID_ARG (iters < 1, blocks_per_sm outside 1..64,
+ * NULL pointer), CUDA. */
+seedq_status seedq_fp64_fma_probe(int64_t iters, int32_t blocks_per_sm, double *out,
+                                  void *cuda_stream, int64_t *fmas);
 
 /* -------------------------------------------------------------- container
  * A file holding a compressed model: the global decoder table (Sec. 3.6, as

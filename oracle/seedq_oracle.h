@@ -86,6 +86,8 @@ typedef struct {
   int rho_uniform; /* 1 when every rho[r] == 1 (all rows share one rung map) */
 } or_factors;
 
+/* Not safe to call from two threads at once: the sort keeps its key in a
+ * file-scope pointer.  The other functions only read their factors. */
 int or_factors_init(or_factors *f, int64_t R, int64_t C, const float *a,
                     const float *rho /* NULL => all ones */);
 void or_factors_free(or_factors *f);

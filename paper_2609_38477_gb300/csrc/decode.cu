@@ -30,7 +30,16 @@ __global__ void __launch_bounds__(256) k_decode(const __grid_constant__ LayerArg
     int32_t bk[kMaxJ];
     for (int j = 0; j < p.J - 1; ++j) bk[j] = __ldg(p.brk + r * (p.J - 1) + j);
     const int g = rung_of(bk, p.J, c);
-    const uint64_t off = __ldg(p.row_off + r) + bits_before(bk, p.J, p.L, p.nb, c);
+    const uint64_t roff = __ldg(p.row_off + r);
+    const uint64_t off = roff + bits_before(bk, p.J, p.L, p.nb, c);
+    // The plan and the bound buffer must agree: the last block of a row ends
+    // at the next row's offset, and the block's three words are readable.
+    // Otherwise flag bit 0 and leave the block's weights unwritten.
+    if (c == p.nb - 1 && off + (uint64_t)p.L[g] != __ldg(p.row_off + r + 1)) atomicOr(p.flags, 1u);
+    if ((off >> 5) + 3 > p.stream_words) {
+      atomicOr(p.flags, 1u);
+      continue;
+    }
     const uint64_t *tab = p.tables + (size_t)p.slot[g] * 512;
     float *Wrow = W + i * p.C;
     const int S = rung_S(p.code[g]);

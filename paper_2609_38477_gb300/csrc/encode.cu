@@ -403,6 +403,23 @@ static int grid_for(int64_t nblocks) {
 
 using namespace seedq;
 
+// fp64 FMA rate probe: eight independent DFMA chains per thread, so the fp64
+// pipe (not latency) bounds it.  Each thread does 8 * iters FMAs.
+__global__ void __launch_bounds__(256) k_fp64_probe(int64_t iters, double seed, double *out) {
+  double v[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) v[i] = seed + (double)(threadIdx.x + i);
+  const double m = 1.0 - 1.0 / 1099511627776.0, c = seed * 1e-9;
+  for (int64_t it = 0; it < iters; ++it) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = __fma_rn(v[i], m, c);
+  }
+  double s = 0.0;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) s += v[i];
+  if (s == 0.123456789) out[0] = s;  // keeps the chains live; never true in practice
+}
+
 extern "C" {
 
 seedq_status seedq_encode_blocks(int32_t S, int32_t k, const float *w, int64_t nblocks, uint32_t *seed,
@@ -442,6 +459,19 @@ seedq_status seedq_pack_stream(const seedq_layer *L, const uint32_t *seed, const
     e = cudaGetLastError();
   }
   return e == cudaSuccess ? SEEDQ_OK : cuda_fail(e);
+}
+
+seedq_status seedq_fp64_fma_probe(int64_t iters, int32_t blocks_per_sm, double *out, void *cuda_stream,
+                                  int64_t *fmas) {
+  if (iters < 1 || blocks_per_sm < 1 || blocks_per_sm > 64 || !out || !fmas) return SEEDQ_ERR_INVALID_ARG;
+  int dev = 0, sms = 0;
+  SEEDQ_CUDA(cudaGetDevice(&dev));
+  SEEDQ_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+  const int grid = sms * blocks_per_sm;
+  k_fp64_probe<<<grid, 256, 0, (cudaStream_t)cuda_stream>>>(iters, 0.5, out);
+  SEEDQ_CUDA(cudaGetLastError());
+  *fmas = (int64_t)grid * 256 * 8 * iters;
+  return SEEDQ_OK;
 }
 
 }  // extern "C"

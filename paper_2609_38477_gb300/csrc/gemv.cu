@@ -244,6 +244,8 @@ __device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t 
     const uint32_t bw[4] = {m0.z, m0.w, m1.x, m1.y};
     uint32_t s_cs, s_ce;
     lane_bits_before(bw, p, cs, ce, s_cs, s_ce);
+    // A row's last stage ends where its record says the row ends.
+    if (ce == nb && s_ce != m1.z) atomicOr(p.flags, 1u);
     // Rung of block cs (breakpoints at or below it) and the next breakpoint.
     int jr0 = 0, nx0 = nb;
 #pragma unroll

@@ -102,13 +102,14 @@ __global__ void k_rowrec(const int32_t *__restrict__ rowperm, const uint64_t *__
        i += (int64_t)gridDim.x * blockDim.x) {
     const int64_t r = rowperm[i];
     const uint64_t off = row_off[r];
+    const uint32_t row_bits = (uint32_t)(row_off[r + 1] - off);
     static_assert(kMaxJ == 9, "the record holds eight breakpoints");
     uint32_t b[kMaxJ - 1];
 #pragma unroll
     for (int j = 0; j < kMaxJ - 1; ++j)
       b[j] = j < J - 1 ? (uint32_t)(uint16_t)brk[r * (J - 1) + j] : 0u;
     rec[2 * i] = make_uint4((uint32_t)off, (uint32_t)(off >> 32), b[0] | (b[1] << 16), b[2] | (b[3] << 16));
-    rec[2 * i + 1] = make_uint4(b[4] | (b[5] << 16), b[6] | (b[7] << 16), 0u, 0u);
+    rec[2 * i + 1] = make_uint4(b[4] | (b[5] << 16), b[6] | (b[7] << 16), row_bits, 0u);
   }
 }
 
@@ -632,6 +633,7 @@ seedq_status seedq_layer_prepare(const seedq_layer_desc *d, const seedq_schedule
   L->args.flags = L->d_flags;
 
   L->args.stream = nullptr;
+  L->args.stream_words = 0;
 
   RungBits rb;
   for (int j = 0; j < kMaxJ; ++j) rb.L[j] = L->args.L[j];
@@ -714,6 +716,16 @@ seedq_status seedq_layer_bind_stream(seedq_layer *L, const void *stream, uint64_
   L->stream = stream;
   L->stream_bytes = bytes;
   L->args.stream = (const uint32_t *)stream;
+  L->args.stream_words = bytes / 4;
+  return SEEDQ_OK;
+}
+
+seedq_status seedq_layer_limit_stream_bytes(seedq_layer *L, uint64_t bytes) {
+  if (!L) return SEEDQ_ERR_INVALID_ARG;
+  if (!L->args.stream) return SEEDQ_ERR_STREAM;
+  if (bytes > L->stream_bytes) return SEEDQ_ERR_INVALID_ARG;
+  L->stream_bytes = bytes;
+  L->args.stream_words = bytes / 4;
   return SEEDQ_OK;
 }
 

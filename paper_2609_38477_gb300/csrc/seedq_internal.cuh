@@ -29,6 +29,7 @@ __host__ __device__ constexpr int rung_K(int code) { return 2 + code % 5; }
 // Everything a kernel needs about one layer, passed by value.
 struct LayerArgs {
   const uint32_t *stream;   // payload words (little-endian bit string)
+  uint64_t stream_words;    // readable 32-bit words of the bound stream buffer
   const uint64_t *row_off;  // R + 1 bit offsets
   const int32_t *brk;       // R x (J-1): first block of row r with rung > j
   const uint64_t *tables;   // nslots x 512 LFSR jump tables
@@ -37,8 +38,9 @@ struct LayerArgs {
   const uint16_t *out_vals; // R x n_out binary16
   const int32_t *rowperm;   // R: order in which rows are grouped 32 to a warp
   const uint4 *rowrec;      // R x 2, at row position i (row rowperm[i]): its bit
-                            // offset (words 0-1) and its breakpoints as int16
-                            // pairs (words 2-5, zero past J - 1)
+                            // offset (words 0-1), its breakpoints as int16
+                            // pairs (words 2-5, zero past J - 1) and its bit
+                            // count (word 6)
   float *xperm;             // C x n: activations in permuted order, weight-major
   int32_t *counters;        // row groups: arrivals of partial sums (0 between calls)
   float *slots;             // max_ctas x 2 x 32 x 16 partial sums of row groups
@@ -348,7 +350,13 @@ __device__ __forceinline__ void reconstruct_rt(uint32_t lo, uint32_t hi, const u
 // the remainder exceeds mb (binary division never lands exactly halfway).  q
 // comes from an estimate of 2^116 / mb (an fp32 reciprocal refined by two
 // Newton steps in fixed point) and is then corrected against the exact
-// 128-bit remainder, so the estimate only has to be within a few units.
+// 128-bit remainder, so the estimate only has to be within a few units.  The
+// method is Newton-Raphson refinement of a reciprocal approximation followed
+// by quotient correction from the exact remainder, as in the literature on
+// division with a precomputed reciprocal (Granlund and Montgomery, "Division
+// by invariant integers using multiplication", PLDI 1994; Markstein, "IA-64
+// and Elementary Functions", 2000).  A GPU test compares it bit for bit with
+// the hardware division on random and edge operands.
 struct DivRecip {
   double b;      // the divisor (for the rare operands handled by hardware division)
   uint64_t d;    // significand of b

@@ -90,6 +90,9 @@ SIGNATURES = {
     "seedq_layer_stream_bits": (C.c_int, [C.c_void_p, C.POINTER(C.c_uint64)]),
     "seedq_stream_bytes_required": (C.c_uint64, [C.c_uint64]),
     "seedq_layer_bind_stream": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint64, C.c_uint64]),
+    "seedq_layer_limit_stream_bytes": (C.c_int, [C.c_void_p, C.c_uint64]),
+    "seedq_fp64_fma_probe": (C.c_int, [C.c_int64, C.c_int32, C.c_void_p, C.c_void_p,
+                                       C.POINTER(C.c_int64)]),
     "seedq_layer_release": (C.c_int, [C.c_void_p]),
     "seedq_decode_weights": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
     "seedq_decode_rows": (C.c_int, [C.c_void_p, C.c_int64, C.c_int64, C.c_void_p, C.c_void_p]),
@@ -236,6 +239,9 @@ class Layer:
         _check(lib().seedq_layer_bind_stream(self.h, _ptr(buf), bits, nbytes), "seedq_layer_bind_stream")
         self._stream_buf = buf
 
+    def limit_stream_bytes(self, nbytes: int):
+        _check(lib().seedq_layer_limit_stream_bytes(self.h, nbytes), "seedq_layer_limit_stream_bytes")
+
     def synth_stream(self, key: int, buf, nbytes: int, stream=None):
         _check(lib().seedq_synth_stream(self.h, key, _ptr(buf), nbytes, _stream(stream)),
                "seedq_synth_stream")
@@ -312,6 +318,14 @@ def encode_blocks(S: int, k: int, w, nblocks: int, seed, E, t, err=None, stream=
     """seedq_encode_blocks: exhaustive seed search of nblocks blocks at rung (S, k)."""
     _check(lib().seedq_encode_blocks(S, k, _ptr(w), nblocks, _ptr(seed), _ptr(E), _ptr(t), _ptr(err),
                                      _stream(stream)), "seedq_encode_blocks")
+
+
+def fp64_fma_probe(iters: int, blocks_per_sm: int, out, stream=None) -> int:
+    """seedq_fp64_fma_probe: launch the fp64 FMA rate probe; returns its FMA count."""
+    n = C.c_int64()
+    _check(lib().seedq_fp64_fma_probe(iters, blocks_per_sm, _ptr(out), _stream(stream), C.byref(n)),
+           "seedq_fp64_fma_probe")
+    return n.value
 
 
 def synth_fp16(key: int, first: int, n: int, m: int, e: int, out, stream=None):

@@ -51,11 +51,19 @@ def otensor(w, i):
     return O.Tensor(t.R, t.C, *W.importance(w, i))
 
 
-def check_y(y, y64, yabs):
+def check_y(y, y64, yabs, cols=28672):
+    """Reading R15's criterion, then the fp32 accumulation bound, which is far
+    tighter: a block adds at most 8 products, a row at most cols/8 block terms
+    in sequence, and at most 32 more additions combine partial sums, so
+    |y - y64| <= (cols/8 + 32) 2^-24 sum|W_hat x| to first order (cols defaults
+    to the widest tensor of the workloads).  A mis-parsed block moves y by about
+    8/cols of sum|W_hat x|, above this bound."""
     y = np.asarray(y, np.float64)
     err = np.abs(y - y64)
     assert err.max() <= TOL * max(np.abs(y64).max(), 1e-30), err.max()
     assert np.all(err <= TOL * yabs + 1e-30), (err / np.maximum(yabs, 1e-30)).max()
+    acc = (cols // 8 + 32) * 2.0 ** -24
+    assert np.all(err <= acc * yabs + 1e-30), (err / np.maximum(yabs, 1e-30)).max()
     return float((err / np.maximum(yabs, 1e-30)).max())
 
 
