@@ -102,17 +102,20 @@ __device__ __forceinline__ int cta_of(const int64_t *cb, int ctas, int64_t u) {
 
 // One block: reconstruct its 8 weights and add scale * sum_i I_i x_b[i] to
 // acc[b].  xc holds the block's activations weight-major, NB per weight
-// (xc[i * NB + b]).  At NB = 1 the products run in the packed halves the
-// reconstruction leaves them in (even and odd weights); at NB >= 2 two batch
-// columns share each packed instruction, in two chains (weights 0-3, 4-7).
+// (xc[i * NB + b]).  The reconstruction leaves (I[2p], I[2p+1]) in the two
+// halves of a packed pair, the odd half 2^Ko times larger (reconstruct_dn).
+// At NB = 1 the products run in those halves, which are added with the odd
+// one scaled back; at NB >= 2 two batch columns share each packed
+// instruction, in one chain over the even and one over the odd weights.
 template <int K, int NB>
 __device__ __forceinline__ void block_fma(const uint32_t (&w)[3], uint32_t sh, const uint64_t *tab,
-                                          const RungRt<K> &rc, const float *xc, float (&acc)[NB]) {
-  const uint32_t lo = __funnelshift_r(w[0], w[1], sh);
+                                          const RungDn<K> &rc, const float *xc, float (&acc)[NB]) {
+  const uint32_t lo = __funnelshift_r(w[0], w[1], sh);  // the shift is taken mod 32
   const uint32_t hi = __funnelshift_r(w[1], w[2], sh);
   uint64_t I2[4];
   float scale;
-  reconstruct_rt2<K>(lo, hi, tab, rc, I2, scale);
+  reconstruct_dn<K>(lo, hi, tab, rc, I2, scale);
+  constexpr float kOdd = 1.0f / (float)(1 << RungDn<K>::Ko);
   if constexpr (NB == 1) {
     const ulonglong2 xa = *reinterpret_cast<const ulonglong2 *>(xc);
     const ulonglong2 xb = *reinterpret_cast<const ulonglong2 *>(xc + 4);
@@ -121,7 +124,7 @@ __device__ __forceinline__ void block_fma(const uint32_t (&w)[3], uint32_t sh, c
     s2 = f2_fma(I2[2], xb.x, s2);
     s2 = f2_fma(I2[3], xb.y, s2);
     const float2 sv = f2_unpack(s2);
-    acc[0] = __fmaf_rn(scale, sv.x + sv.y, acc[0]);
+    acc[0] = __fmaf_rn(scale, __fmaf_rn(sv.y, kOdd, sv.x), acc[0]);
   } else {
     const uint64_t *x2 = reinterpret_cast<const uint64_t *>(xc);  // pairs of batch columns
     uint64_t Ip[8];
@@ -131,17 +134,17 @@ __device__ __forceinline__ void block_fma(const uint32_t (&w)[3], uint32_t sh, c
       Ip[2 * p] = f2_pack(v.x, v.x);
       Ip[2 * p + 1] = f2_pack(v.y, v.y);
     }
-    const uint64_t sp = f2_pack(scale, scale);
+    const uint64_t sp = f2_pack(scale, scale), ko = f2_pack(kOdd, kOdd);
 #pragma unroll
     for (int q = 0; q < NB / 2; ++q) {
-      uint64_t s0 = f2_mul(Ip[0], x2[0 * (NB / 2) + q]), s1 = f2_mul(Ip[4], x2[4 * (NB / 2) + q]);
-      s0 = f2_fma(Ip[1], x2[1 * (NB / 2) + q], s0);
-      s1 = f2_fma(Ip[5], x2[5 * (NB / 2) + q], s1);
+      uint64_t s0 = f2_mul(Ip[0], x2[0 * (NB / 2) + q]), s1 = f2_mul(Ip[1], x2[1 * (NB / 2) + q]);
       s0 = f2_fma(Ip[2], x2[2 * (NB / 2) + q], s0);
-      s1 = f2_fma(Ip[6], x2[6 * (NB / 2) + q], s1);
-      s0 = f2_fma(Ip[3], x2[3 * (NB / 2) + q], s0);
+      s1 = f2_fma(Ip[3], x2[3 * (NB / 2) + q], s1);
+      s0 = f2_fma(Ip[4], x2[4 * (NB / 2) + q], s0);
+      s1 = f2_fma(Ip[5], x2[5 * (NB / 2) + q], s1);
+      s0 = f2_fma(Ip[6], x2[6 * (NB / 2) + q], s0);
       s1 = f2_fma(Ip[7], x2[7 * (NB / 2) + q], s1);
-      const uint64_t a = f2_fma(sp, f2_add(s0, s1), f2_pack(acc[2 * q], acc[2 * q + 1]));
+      const uint64_t a = f2_fma(sp, f2_fma(s1, ko, s0), f2_pack(acc[2 * q], acc[2 * q + 1]));
       acc[2 * q] = __uint_as_float((uint32_t)a);
       acc[2 * q + 1] = __uint_as_float((uint32_t)(a >> 32));
     }
@@ -153,7 +156,7 @@ __device__ __forceinline__ void run_cols(int S, const uint32_t *rowbuf, uint32_t
                                          const uint64_t *tab, const float *xc,
                                          uint32_t z, float (&acc)[NB]) {
   const uint32_t L = (uint32_t)(S + 4 * K + 4);
-  const RungRt<K> rc(S, z);
+  const RungDn<K> rc(S, z);
   uint32_t w[3];
   {
     const uint32_t *q = rowbuf + (pos >> 5);
@@ -163,7 +166,7 @@ __device__ __forceinline__ void run_cols(int S, const uint32_t *rowbuf, uint32_t
   }
   for (int i = 0; i < n; ++i) {
     const uint32_t cur[3] = {w[0], w[1], w[2]};
-    const uint32_t sh = pos & 31;
+    const uint32_t sh = pos;
     pos += L;
     if (i + 1 < n) {
       const uint32_t *q = rowbuf + (pos >> 5);

@@ -340,6 +340,130 @@ __device__ __forceinline__ void reconstruct_rt(uint32_t lo, uint32_t hi, const u
   }
 }
 
+// ------------------------------------- reconstruction with subnormal states
+//
+// The same exact integers I[i] of Eq. codec, with fewer logic instructions
+// (the fused kernel's form; reconstruct_rt above stays the decoder's).
+//
+// A 32-bit word whose sign and exponent bits are zero is the float
+// m * 2^-149, m its 23-bit mantissa field.  So a state x_n lying at bit
+// offset o of a 32-bit window of the sequence (bits [o, o + S), o + S <= 23),
+// masked out of the window by a single AND, is the float x_n * 2^(o - 149):
+// no exponent has to be inserted and the state need not sit at a fixed
+// position.  One window thus serves every state that starts in its first
+// 24 - S bits, and Q is used as the tables return it (no shift into exponent
+// position):
+//   K <= 4: the window at bit 2pK holds the 2K states of weights 2p and 2p+1
+//           (offsets j and K + j; 2K + S <= 24 for S <= 16);
+//   K >= 5: the window at bit iK holds the K states of weight i (offset j).
+//
+// The offsets go into the coefficients: tf_j = t_j * 2^(M - j) (M = 108) comes
+// straight from the 4-bit field read under a larger exponent, so
+// tf_j * x_n 2^(j - 149) = t_j x_n u with u = 2^(M - 149) = 2^-41 for a weight
+// at offset j, and 2^K times that for the odd weight of a shared window.
+// Every product is exact, every partial sum of a chain is an integer multiple
+// of its unit below 2^24 units (|partial| <= 12 K 2^S < 2^23 for S <= 16,
+// K <= 6), so each chain yields its I exactly:
+//   Ip[p] = (I[2p] u, I[2p+1] u 2^Ko), Ko = K for K <= 4, else 0,
+// and scale = 2^(E - S + 1) / u.  The FMAs keep subnormal operands (no .ftz).
+// Scaling by powers of two changes no rounding, so a product with x rounds as
+// it would on the unscaled I (unless |x| < 2^-85, where u I x is subnormal).
+constexpr int kDnM = 108;
+
+__host__ __device__ constexpr int field_pos(int j) { return (4 + 4 * j <= 19) ? 4 + 4 * j : 4 + 4 * j - 16; }
+// The float read from field j when t_j = 0 (field value 8 after the XOR):
+// 2^(131 - P - j) + 8 * 2^(M - j); any t_j reads as that plus t_j 2^(M - j).
+__host__ __device__ constexpr uint32_t dn_tbits(int j) {
+  return (8u << field_pos(j)) | ((uint32_t)(150 + kDnM - field_pos(j) - j) << 23);
+}
+static_assert(150 + kDnM - 4 <= 254, "coefficient exponent out of range");
+
+template <int K>
+struct RungDn {
+  static constexpr bool kPair = 2 * K + 16 <= 24;
+  static constexpr int Ko = kPair ? K : 0;
+  uint32_t S;
+  uint32_t e_msk, e_x, sc;      // E field (at bit 0) and the scale's exponent offset
+  uint32_t t_msk[K], t_x[K];    // t_j fields
+  uint32_t m_e[K];              // state masks: offset j
+  uint32_t m_o[kPair ? K : 1];  // offset K + j (odd weight of a shared window)
+  uint64_t cinit2[K];           // (-2^(S+j-150), -2^(S+j-150+Ko)): the centring -2^(S-1) t_j u
+  __device__ __forceinline__ RungDn(int S_, uint32_t z) {
+    S = (uint32_t)S_;
+    e_msk = 15u ^ z;
+    e_x = 8u ^ z;
+    sc = ((uint32_t)(120 + 149 - kDnM - S_) << 23) ^ z;
+    const uint32_t ms = (1u << S_) - 1u;
+#pragma unroll
+    for (int j = 0; j < K; ++j) {
+      t_msk[j] = (15u << field_pos(j)) ^ z;
+      t_x[j] = dn_tbits(j) ^ z;
+      m_e[j] = (ms << j) ^ z;
+      if constexpr (kPair) m_o[j] = (ms << (K + j)) ^ z;
+      // Subnormal: S + j - 1 + Ko <= 22.
+      const uint32_t ce = 0x80000000u | (1u << (S_ + j - 1)), co = 0x80000000u | (1u << (S_ + j - 1 + Ko));
+      cinit2[j] = ((uint64_t)(co ^ z) << 32) | (uint64_t)(ce ^ z);
+    }
+  }
+};
+
+// Bits [N, N + 32) of Q = (qhi:qlo), zero past bit 63 (0 <= N < 64).
+template <int N>
+__device__ __forceinline__ uint32_t qwin2(uint32_t qlo, uint32_t qhi) {
+  if constexpr (N == 0) return qlo;
+  else if constexpr (N < 32) return __funnelshift_r(qlo, qhi, N);
+  else if constexpr (N == 32) return qhi;
+  else return qhi >> (N - 32);
+}
+
+template <int K, int P, int J>
+__device__ __forceinline__ uint64_t dn_chain(uint32_t qlo, uint32_t qhi, const RungDn<K> &rc,
+                                             const uint64_t (&tf2)[K], uint64_t acc) {
+  if constexpr (J >= K) {
+    return acc;
+  } else {
+    uint32_t se, so;
+    if constexpr (RungDn<K>::kPair) {
+      const uint32_t w = qwin2<2 * P * K>(qlo, qhi);
+      se = w & rc.m_e[J];
+      so = w & rc.m_o[J];
+    } else {
+      se = qwin2<2 * P * K>(qlo, qhi) & rc.m_e[J];
+      so = qwin2<(2 * P + 1) * K>(qlo, qhi) & rc.m_e[J];
+    }
+    acc = f2_fma(tf2[J], f2_pack(__uint_as_float(se), __uint_as_float(so)), acc);
+    return dn_chain<K, P, J + 1>(qlo, qhi, rc, tf2, acc);
+  }
+}
+
+// lo, hi: the block's 64 field bits starting at its first bit.
+template <int K>
+__device__ __forceinline__ void reconstruct_dn(uint32_t lo, uint32_t hi, const uint64_t *tab,
+                                               const RungDn<K> &rc, uint64_t (&Ip)[4], float &scale) {
+  // For S = 8 the second table half is all zero, so both lookups are always valid.
+  const uint64_t Q = tab[lo & 255u] ^ tab[256 + __byte_perm(lo, 0, 0x4441)];
+  const uint32_t qlo = (uint32_t)Q, qhi = (uint32_t)(Q >> 32);
+  const uint32_t f = __funnelshift_r(lo, hi, rc.S);
+  const uint32_t e8 = lop_and_xor(f, rc.e_msk, rc.e_x);
+  scale = __uint_as_float(e8 * (1u << 23) + rc.sc);
+  uint64_t tf2[K];
+  uint32_t f2 = 0;
+  if constexpr (K > 4) f2 = f >> 16;
+#pragma unroll
+  for (int j = 0; j < K; ++j) {
+    const uint32_t w = (4 + 4 * j <= 19) ? f : f2;
+    const float tf = __uint_as_float(lop_and_xor(w, rc.t_msk[j], rc.t_x[j])) - __uint_as_float(dn_tbits(j));
+    tf2[j] = f2_pack(tf, tf);
+  }
+  uint64_t init2 = f2_mul(tf2[0], rc.cinit2[0]);
+#pragma unroll
+  for (int j = 1; j < K; ++j) init2 = f2_fma(tf2[j], rc.cinit2[j], init2);
+  Ip[0] = dn_chain<K, 0, 0>(qlo, qhi, rc, tf2, init2);
+  Ip[1] = dn_chain<K, 1, 0>(qlo, qhi, rc, tf2, init2);
+  Ip[2] = dn_chain<K, 2, 0>(qlo, qhi, rc, tf2, init2);
+  Ip[3] = dn_chain<K, 3, 0>(qlo, qhi, rc, tf2, init2);
+}
+
 
 // ------------------------------------------------- fp64 division, integer pipes
 //
