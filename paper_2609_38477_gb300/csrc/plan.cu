@@ -38,53 +38,122 @@ static const uint32_t kTaps[17] = {0, 0, 0, 0, 0, 0, 0, 0,
 
 // ------------------------------------------------------------ plan kernels
 
-// Stable ascending rank of a: perm[rank(i)] = i with ties broken by index
-// (Sec. 3.3: channels sorted by a before blocking).  blk: this block's index
-// among the ceil(C / blockDim.x) blocks of the tensor.
-__device__ __forceinline__ void perm_block(const float *__restrict__ a, int C, int blk,
-                                           int32_t *__restrict__ perm) {
-  __shared__ float tile[1024];
-  const int i = blk * blockDim.x + threadIdx.x;
-  const float ai = (i < C) ? a[i] : 0.f;
-  int rank = 0;
-  for (int base = 0; base < C; base += 1024) {
-    __syncthreads();
-    for (int t = threadIdx.x; t < 1024; t += blockDim.x)
-      tile[t] = (base + t < C) ? a[base + t] : 0.f;
-    __syncthreads();
-    const int n = min(1024, C - base);
-    for (int t = 0; t < n; ++t) {
-      const float v = tile[t];
-      rank += (v < ai || (v == ai && base + t < i)) ? 1 : 0;
-    }
-  }
-  if (i < C) perm[rank] = i;
+// Stable ranking of n keys in O(n log n): every chunk of kRankChunk keys is
+// sorted by (key, index) in shared memory (bitonic network), then each key's
+// rank is the number of entries below it in every sorted chunk (a binary
+// search per chunk), and out[rank] = its index.  The order is ascending keys
+// (kDesc: descending), ties by ascending index:
+//   perm:    columns by ascending a (Sec. 3.3: channels sorted by a before
+//            blocking), perm[rank] = column;
+//   rowperm: the fused kernel's row order, rows by decreasing rho, so rows
+//            with equal or nearby rung breakpoints (monotone in imp = abar *
+//            rho) share a warp; with no row factor the natural order is kept.
+// One launch serves several jobs (blocks located by binary search over their
+// first-block numbers).
+constexpr int kRankChunk = 1024;
+
+template <typename K>
+struct RankJob {
+  const K *key;
+  int32_t *out;     // n: out[rank] = index
+  K *skey;          // scratch: n keys in sorted chunks
+  int32_t *sidx;    // scratch: their indices
+  int32_t n;
+  int32_t sblk0;    // first block of this job in the sort launch (one per chunk)
+  int32_t rblk0;    // first block of this job in the rank launch (256 keys each)
+};
+
+template <typename K, bool kDesc>
+__device__ __forceinline__ bool rank_less(K ka, int32_t ia, K kb, int32_t ib) {
+  // Padding entries (index -1) sort after every key.
+  if (ia < 0) return false;
+  if (ib < 0) return true;
+  if (ka != kb) return kDesc ? ka > kb : ka < kb;
+  return ia < ib;
 }
 
-__global__ void k_perm(const float *__restrict__ a, int C, int32_t *__restrict__ perm) {
-  perm_block(a, C, blockIdx.x, perm);
+template <typename K>
+__device__ __forceinline__ int rank_job(const RankJob<K> *jobs, int nj, int b, bool sort_launch) {
+  int lo = 0, hi = nj - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if ((sort_launch ? jobs[mid].sblk0 : jobs[mid].rblk0) <= b) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
 }
 
-// Row order for the fused kernel: rows with equal or nearby rung breakpoints
-// share a warp.  Breakpoints are monotone in the row factor (imp = abar * rho),
-// so rows are ranked by decreasing rho (ties by index); with no row factor every
-// row has the same breakpoints and the natural order is kept.
-__global__ void k_rowrank(const double *__restrict__ rho, int R, int32_t *__restrict__ rowperm) {
-  __shared__ double tile[1024];
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  const double ri = (i < R) ? rho[i] : 0.0;
-  int rank = 0;
-  for (int base = 0; base < R; base += 1024) {
-    __syncthreads();
-    for (int t = threadIdx.x; t < 1024; t += blockDim.x) tile[t] = (base + t < R) ? rho[base + t] : 0.0;
-    __syncthreads();
-    const int n = min(1024, R - base);
-    for (int t = 0; t < n; ++t) {
-      const double v = tile[t];
-      rank += (v > ri || (v == ri && base + t < i)) ? 1 : 0;
+template <typename K, bool kDesc>
+__global__ void __launch_bounds__(kRankChunk / 2) k_chunk_sort(const RankJob<K> *__restrict__ jobs, int nj) {
+  __shared__ K sk[kRankChunk];
+  __shared__ int32_t si[kRankChunk];
+  const RankJob<K> &J = jobs[rank_job(jobs, nj, blockIdx.x, true)];
+  const int base = (blockIdx.x - J.sblk0) * kRankChunk;
+  for (int t = threadIdx.x; t < kRankChunk; t += blockDim.x) {
+    const int i = base + t;
+    sk[t] = i < J.n ? J.key[i] : K(0);
+    si[t] = i < J.n ? i : -1;
+  }
+  __syncthreads();
+  for (int k = 2; k <= kRankChunk; k <<= 1) {
+    for (int j = k >> 1; j > 0; j >>= 1) {
+      const int t = threadIdx.x;
+      const int i = ((t & ~(j - 1)) << 1) | (t & (j - 1)), l = i + j;
+      const bool up = (i & k) == 0;
+      const bool sw = up ? rank_less<K, kDesc>(sk[l], si[l], sk[i], si[i])
+                         : rank_less<K, kDesc>(sk[i], si[i], sk[l], si[l]);
+      if (sw) {
+        const K tk = sk[i];
+        sk[i] = sk[l];
+        sk[l] = tk;
+        const int32_t ti = si[i];
+        si[i] = si[l];
+        si[l] = ti;
+      }
+      __syncthreads();
     }
   }
-  if (i < R) rowperm[rank] = i;
+  for (int t = threadIdx.x; t < kRankChunk && base + t < J.n; t += blockDim.x) {
+    J.skey[base + t] = sk[t];
+    J.sidx[base + t] = si[t];
+  }
+}
+
+template <typename K, bool kDesc>
+__global__ void __launch_bounds__(256) k_chunk_rank(const RankJob<K> *__restrict__ jobs, int nj) {
+  const RankJob<K> &J = jobs[rank_job(jobs, nj, blockIdx.x, false)];
+  const int i = (blockIdx.x - J.rblk0) * 256 + threadIdx.x;
+  if (i >= J.n) return;
+  const K ki = J.key[i];
+  int rank = 0;
+  for (int c0 = 0; c0 < J.n; c0 += kRankChunk) {
+    int lo = 0, hi = min(kRankChunk, J.n - c0);
+    while (lo < hi) {
+      const int mid = (lo + hi) >> 1;
+      if (rank_less<K, kDesc>(J.skey[c0 + mid], J.sidx[c0 + mid], ki, i)) lo = mid + 1;
+      else hi = mid;
+    }
+    rank += lo;
+  }
+  J.out[rank] = i;
+}
+
+// Launches the two kernels over nj jobs whose descriptors (with block numbers
+// filled in by this function) go to d_jobs.
+template <typename K, bool kDesc>
+static cudaError_t launch_rank(RankJob<K> *h_jobs, int nj, RankJob<K> *d_jobs, cudaStream_t st) {
+  int sb = 0, rbk = 0;
+  for (int t = 0; t < nj; ++t) {
+    h_jobs[t].sblk0 = sb;
+    h_jobs[t].rblk0 = rbk;
+    sb += (h_jobs[t].n + kRankChunk - 1) / kRankChunk;
+    rbk += (h_jobs[t].n + 255) / 256;
+  }
+  cudaError_t e = cudaMemcpyAsync(d_jobs, h_jobs, sizeof(RankJob<K>) * nj, cudaMemcpyHostToDevice, st);
+  if (e != cudaSuccess || sb == 0) return e;
+  k_chunk_sort<K, kDesc><<<sb, kRankChunk / 2, 0, st>>>(d_jobs, nj);
+  k_chunk_rank<K, kDesc><<<rbk, 256, 0, st>>>(d_jobs, nj);
+  return cudaGetLastError();
 }
 
 __global__ void k_iota(int64_t n, int32_t *__restrict__ out) {
@@ -172,19 +241,7 @@ struct FacJob {
   double *rho;          // R
   int64_t R;
   int32_t C;
-  int32_t blk0;         // first block of this tensor in k_perm_multi
 };
-
-__global__ void k_perm_multi(const FacJob *__restrict__ jobs, int nt) {
-  int lo = 0, hi = nt - 1;
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (jobs[mid].blk0 <= (int)blockIdx.x) lo = mid;
-    else hi = mid - 1;
-  }
-  const FacJob &J = jobs[lo];
-  perm_block(J.a, J.C, blockIdx.x - J.blk0, J.perm);
-}
 
 __global__ void k_factors_multi(const FacJob *__restrict__ jobs) {
   const FacJob &J = jobs[blockIdx.x];
@@ -637,12 +694,27 @@ seedq_status seedq_layer_prepare(const seedq_layer_desc *d, const seedq_schedule
 
   RungBits rb;
   for (int j = 0; j < kMaxJ; ++j) rb.L[j] = L->args.L[j];
-  cudaError_t e = cudaMemsetAsync(L->d_flags, 0, sizeof(uint32_t), st);
+  bool rho_uniform = true;
+  if (d->rho)
+    for (int64_t r = 1; r < R; ++r) rho_uniform &= (d->rho[r] == d->rho[0]);
+  const bool rank_rows = !rho_uniform && R <= 65536;
+  // Scratch of the stable rankings (columns by a, rows by rho), freed below.
+  uint8_t *scr = nullptr;
+  const size_t scr_cols = (size_t)C * 8, scr_rows = rank_rows ? (size_t)R * 16 : 0;
+  const size_t scr_jobs = sizeof(RankJob<float>) + sizeof(RankJob<double>);
+  cudaError_t e = cudaMalloc((void **)&scr, scr_cols + scr_rows + scr_jobs);
+  if (e != cudaSuccess) {
+    free_layer(L);
+    return cuda_fail(e);
+  }
+  if (e == cudaSuccess) e = cudaMemsetAsync(L->d_flags, 0, sizeof(uint32_t), st);
   if (e == cudaSuccess) e = cudaMemcpyAsync(L->d_a_in, d->a, sizeof(float) * C, cudaMemcpyHostToDevice, st);
   if (e == cudaSuccess && d->rho)
     e = cudaMemcpyAsync(L->d_rho_in, d->rho, sizeof(float) * R, cudaMemcpyHostToDevice, st);
   if (e == cudaSuccess) {
-    k_perm<<<(int)((C + 255) / 256), 256, 0, st>>>(L->d_a_in, (int)C, L->d_perm);
+    RankJob<float> jc{L->d_a_in, L->d_perm, reinterpret_cast<float *>(scr),
+                      reinterpret_cast<int32_t *>(scr + (size_t)C * 4), (int32_t)C, 0, 0};
+    e = launch_rank<float, false>(&jc, 1, reinterpret_cast<RankJob<float> *>(scr + scr_cols + scr_rows), st);
     k_invperm<<<(int)((C + 255) / 256), 256, 0, st>>>(L->d_perm, (int)C, L->d_invperm);
     k_abar<<<1, 1024, 0, st>>>(L->d_a_in, L->d_perm, nb, L->d_abar);
     k_rho<<<1, 1024, 0, st>>>(L->d_rho_in, R, L->d_rho);
@@ -659,13 +731,13 @@ seedq_status seedq_layer_prepare(const seedq_layer_desc *d, const seedq_schedule
     }
     k_scan<<<1, 1024, 0, st>>>(R, J, nb, J > 1 ? s->j_tie : -1, d->tie_count, rb, L->d_brk,
                                L->d_tcnt, L->d_row_off, L->d_summary);
-    bool rho_uniform = true;
-    if (d->rho)
-      for (int64_t r = 1; r < R; ++r) rho_uniform &= (d->rho[r] == d->rho[0]);
-    if (rho_uniform || R > 65536) {
+    if (!rank_rows) {
       k_iota<<<(int)((R + 255) / 256 < 4096 ? (R + 255) / 256 : 4096), 256, 0, st>>>(R, L->d_rowperm);
-    } else {
-      k_rowrank<<<(int)((R + 255) / 256), 256, 0, st>>>(L->d_rho, (int)R, L->d_rowperm);
+    } else if (e == cudaSuccess) {
+      RankJob<double> jr{L->d_rho, L->d_rowperm, reinterpret_cast<double *>(scr + scr_cols),
+                         reinterpret_cast<int32_t *>(scr + scr_cols + (size_t)R * 8), (int32_t)R, 0, 0};
+      e = launch_rank<double, true>(
+          &jr, 1, reinterpret_cast<RankJob<double> *>(scr + scr_cols + scr_rows + sizeof(RankJob<float>)), st);
     }
     k_rowrec<<<(int)((R + 255) / 256 < 4096 ? (R + 255) / 256 : 4096), 256, 0, st>>>(
         L->d_rowperm, L->d_row_off, L->d_brk, J, R, L->d_rowrec);
@@ -675,6 +747,8 @@ seedq_status seedq_layer_prepare(const seedq_layer_desc *d, const seedq_schedule
   uint64_t summary[2] = {0, 0};
   if (e == cudaSuccess) e = cudaMemcpyAsync(summary, L->d_summary, sizeof summary, cudaMemcpyDeviceToHost, st);
   if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e == cudaSuccess) e = cudaFree(scr);
+  else cudaFree(scr);
   if (e != cudaSuccess) {
     free_layer(L);
     return cuda_fail(e);
@@ -1062,13 +1136,12 @@ extern "C" seedq_status seedq_allocate(const seedq_factor_desc *tensors, int32_t
     owned.push_back(p);
     return p;
   };
-  int64_t n_a = 0, n_rho = 0, n_rows = 0, n_nb = 0, blocks = 0;
+  int64_t n_a = 0, n_rho = 0, n_rows = 0, n_nb = 0;
   for (int t = 0; t < count; ++t) {
     n_a += tensors[t].cols;
     n_rho += tensors[t].rho ? tensors[t].rows : 0;
     n_rows += tensors[t].rows;
     n_nb += tensors[t].cols / 8;
-    blocks += (tensors[t].cols + 255) / 256;
   }
   std::vector<float> h_in((size_t)(n_a + n_rho));
   float *d_in = (float *)dalloc(sizeof(float) * (size_t)(n_a + n_rho));
@@ -1076,7 +1149,12 @@ extern "C" seedq_status seedq_allocate(const seedq_factor_desc *tensors, int32_t
   double *d_abar = (double *)dalloc(sizeof(double) * (size_t)n_nb);
   double *d_rho = (double *)dalloc(sizeof(double) * (size_t)n_rows);
   FacJob *d_jobs = (FacJob *)dalloc(sizeof(FacJob) * count);
-  if (!d_in || !d_perm || !d_abar || !d_rho || !d_jobs) {
+  // Stable column rankings of all tensors in one sort and one rank launch.
+  float *d_skey = (float *)dalloc(sizeof(float) * (size_t)n_a);
+  int32_t *d_sidx = (int32_t *)dalloc(sizeof(int32_t) * (size_t)n_a);
+  RankJob<float> *d_rjobs = (RankJob<float> *)dalloc(sizeof(RankJob<float>) * count);
+  std::vector<RankJob<float>> hr(count);
+  if (!d_in || !d_perm || !d_abar || !d_rho || !d_jobs || !d_skey || !d_sidx || !d_rjobs) {
     cleanup();
     return SEEDQ_ERR_NOMEM;
   }
@@ -1085,7 +1163,6 @@ extern "C" seedq_status seedq_allocate(const seedq_factor_desc *tensors, int32_t
   int64_t rows_total = 0;
   {
     int64_t oa = 0, orh = n_a, orow = 0, onb = 0;
-    int32_t b0 = 0;
     for (int t = 0; t < count; ++t) {
       const seedq_factor_desc &d = tensors[t];
       memcpy(h_in.data() + oa, d.a, sizeof(float) * d.cols);
@@ -1096,11 +1173,11 @@ extern "C" seedq_status seedq_allocate(const seedq_factor_desc *tensors, int32_t
         orh += d.rows;
       }
       hj[t] = FacJob{d_in + oa, rho_dev, d_perm + oa, d_abar + onb, d_rho + orow, d.rows,
-                     (int32_t)d.cols, b0};
+                     (int32_t)d.cols};
+      hr[t] = RankJob<float>{d_in + oa, d_perm + oa, d_skey + oa, d_sidx + oa, (int32_t)d.cols, 0, 0};
       ht[t] = AllocTensor{d_abar + onb, d_rho + orow, d.rows, rows_total, d.rho ? (int32_t)d.rows : 1,
                           (int32_t)(d.cols / 8)};
       rows_total += ht[t].nrows;
-      b0 += (int32_t)((d.cols + 255) / 256);
       oa += d.cols;
       orow += d.rows;
       onb += d.cols / 8;
@@ -1111,8 +1188,8 @@ extern "C" seedq_status seedq_allocate(const seedq_factor_desc *tensors, int32_t
                                     cudaMemcpyHostToDevice, st);
     if (e == cudaSuccess)
       e = cudaMemcpyAsync(d_jobs, hj.data(), sizeof(FacJob) * count, cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess) e = launch_rank<float, false>(hr.data(), count, d_rjobs, st);
     if (e == cudaSuccess) {
-      k_perm_multi<<<(int)blocks, 256, 0, st>>>(d_jobs, count);
       k_factors_multi<<<count, 1024, 0, st>>>(d_jobs);
       e = cudaGetLastError();
     }
