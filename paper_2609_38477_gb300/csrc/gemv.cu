@@ -490,10 +490,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ Mu
     // The output rows of the round, loaded now (thread t < 32 np: row t % 32
     // of piece t / 32): the loads complete during the round; volatile keeps
     // them ahead of the round's copies.
+    // (From the descriptor in the parameter block or device memory: for a layer
+    // set the shared copy sT is still being written by other threads here.)
     __shared__ int32_t srow[8 * 32];
     int32_t crow = -1;
-    if (ck < np && cg * 32 + cln < p.R) {
-      const int32_t *ap = p.rowperm + cg * 32 + cln;
+    const int32_t *trowperm = tens[ti].p.rowperm;
+    if (ck < np && cg * 32 + cln < tens[ti].p.R) {
+      const int32_t *ap = trowperm + cg * 32 + cln;
       asm volatile("{\n\t.reg .u64 ga;\n\tcvta.to.global.u64 ga, %1;\n\tld.global.nc.b32 %0, [ga];\n\t}"
                    : "=r"(crow) : "l"(ap));
     }
