@@ -36,6 +36,8 @@
 #include <string.h>
 
 #include <algorithm>
+#include <map>
+#include <mutex>
 #include <vector>
 
 #include "cp_async.cuh"
@@ -52,7 +54,6 @@ constexpr int kPhases = kCT / 4;               // row phases (4 threads x 8 colu
 constexpr int kUnroll = 8;                     // rows per thread per stage
 constexpr int kStageRows = kUnroll * kPhases;  // 512
 constexpr int kRing = 3;                       // stages in the ring
-constexpr int kItemsPerCta = 1;                // work items per CTA a launch aims for
 constexpr int kHS = 257;                       // histogram row stride (bank spread)
 constexpr int kGH = 64;                        // Gauss-Hermite nodes
 constexpr int kMaxJobs = 4;
@@ -907,15 +908,68 @@ void gauss_hermite(int n, double *x, double *w) {
 
 bool aligned16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
 
-// Slab height of a launch: about kItemsPerCta items per resident CTA, in
-// multiples of kStageRows rows.
-int64_t slab_rows_for(int64_t row_tiles, int ctas) {
-  int64_t h = row_tiles / ((int64_t)kItemsPerCta * ctas);
-  h = (h + kStageRows - 1) / kStageRows * kStageRows;
-  // At most 2048 rows per thread and item, so the FP16 counts stay exact.
-  return h < kStageRows ? kStageRows : std::min<int64_t>(h, 2048 * kPhases);
-}
+// Work items of a job for slab height h: one per (slab, tile).
 int64_t items_of(int64_t R, int64_t C, int64_t h) { return (C / kTC) * ((R + h - 1) / h); }
+
+// Rows per work item of one launch: among the slab heights (multiples of
+// kStageRows, at most 2048 rows per thread and item so the FP16 counts stay
+// exact), the one whose assignment of items to CTAs (item i to CTA i mod the
+// grid, items job by job and slab-major within a job, as the kernel takes
+// them) leaves the smallest busiest CTA, each item counting its rows plus
+// kItemRows for its fixed work (first-stage maxima, end reductions, record,
+// the ring refill across the item boundary).  kItemRows is set by
+// measurement: whole passes over the Llama-2-7B and Llama-3-8B shapes took
+// 9.39 / 8.87 ms at 256, 7.13 / 7.69 at 768, 7.09 / 7.49 at 2048 and
+// 6.93 / 7.41 at 3072 (the choices do not change from 3072 to 4096), against
+// 7.79 / 8.40 with about one item per resident CTA.  Launches of one shape
+// recur every layer, so the choice is cached per shape.
+constexpr int64_t kItemRows = 3072;
+
+int64_t slab_rows_for(const ColArgs &A, int ctas) {
+  std::vector<int64_t> key{(int64_t)ctas};
+  int64_t maxR = 0;
+  for (int i = 0; i < A.njobs; ++i) {
+    key.push_back(A.j[i].R);
+    key.push_back(A.j[i].C);
+    maxR = std::max<int64_t>(maxR, A.j[i].R);
+  }
+  static std::mutex mu;
+  static std::map<std::vector<int64_t>, int64_t> cache;
+  {
+    std::lock_guard<std::mutex> lk(mu);
+    const auto it = cache.find(key);
+    if (it != cache.end()) return it->second;
+  }
+  const int64_t hmax = std::min<int64_t>((maxR + kStageRows - 1) / kStageRows * kStageRows, 2048 * kPhases);
+  std::vector<int64_t> load(ctas);
+  int64_t best_h = kStageRows, best = -1;
+  int64_t last_slabs = -1;
+  for (int64_t h = kStageRows; h <= hmax; h += kStageRows) {
+    const int64_t slabs0 = (maxR + h - 1) / h;
+    if (slabs0 == last_slabs) continue;  // same split of the tallest job as a smaller h
+    last_slabs = slabs0;
+    int64_t items = 0;
+    for (int i = 0; i < A.njobs; ++i) items += items_of(A.j[i].R, A.j[i].C, h);
+    const int64_t G = std::min<int64_t>(items, ctas);
+    std::fill(load.begin(), load.end(), 0);
+    int64_t i = 0;
+    for (int jb = 0; jb < A.njobs; ++jb) {
+      const int64_t R = A.j[jb].R, tiles = A.j[jb].C / kTC, sl = (R + h - 1) / h;
+      for (int64_t s = 0; s < sl; ++s) {
+        const int64_t rows = std::min<int64_t>(h, R - s * h) + kItemRows;
+        for (int64_t t = 0; t < tiles; ++t, ++i) load[i % G] += rows;
+      }
+    }
+    const int64_t m = *std::max_element(load.begin(), load.begin() + G);
+    if (best < 0 || m < best) {
+      best = m;
+      best_h = h;
+    }
+  }
+  std::lock_guard<std::mutex> lk(mu);
+  cache[key] = best_h;
+  return best_h;
+}
 
 // Device scratch of the column pass: one record per work item and one arrival
 // counter per tile (zero between launches).
@@ -937,9 +991,7 @@ int resident_ctas() {
 }
 
 seedq_status launch_cols(ColArgs &A, const ColScratch &S, cudaStream_t st) {
-  int64_t row_tiles = 0;
-  for (int i = 0; i < A.njobs; ++i) row_tiles += A.j[i].R * (A.j[i].C / kTC);
-  const int64_t h = slab_rows_for(row_tiles, S.ctas);
+  const int64_t h = slab_rows_for(A, S.ctas);
   int64_t items = 0, tiles = 0;
   for (int i = 0; i < A.njobs; ++i) {
     ColJob &J = A.j[i];
