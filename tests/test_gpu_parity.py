@@ -317,6 +317,48 @@ def test_edge_cases(case):
     L.release()
 
 
+TIES = [
+    # R, C, number of distinct a values, number of distinct rho values
+    (3, 1024, 1, 0),      # every channel tied: identity order, one whole sort chunk
+    (1030, 1032, 3, 3),   # one chunk plus a 8-key tail; rows ranked by tied rho
+    (257, 3000, 2, 2),    # three chunks, ragged last one
+    (64, 4104, 5, 1),     # five chunks; rho all equal after its unit mean
+]
+
+
+@pytest.mark.parametrize("case", range(len(TIES)))
+def test_ranking_ties(case):
+    """Sec. 3.3 sorts channels ascending by a with ties by channel index, and
+    the rows are ordered by rho; with few distinct values nearly every key is
+    tied, across the boundaries of the device's 1024-key sort chunks."""
+    R, Cc, na, nr = TIES[case]
+    rng = np.random.default_rng(100 + case)
+    a = rng.choice(np.array([0.5, 1.0, 2.0, 3.0, 0.25], np.float32)[:na], Cc)
+    rh = None if nr == 0 else rng.choice(np.array([0.8, 1.0, 1.25], np.float32)[:nr], R)
+    ot = O.Tensor(R, Cc, a, rh)
+    s = O.Sched([(8, 2), (12, 3), (16, 4)], [0.9, 1.2], -1, 0.1)
+    ost, bits = ot.synth_pack(s, 0, 4242 + case)
+    L = _gpu_layer(R, Cc, a, rh, s, 0, ost, bits, None, None)
+    assert np.array_equal(L.perm(), np.argsort(a, kind="stable"))
+    assert np.array_equal(L.rung_map(), ot.rung_rows(s, 0))
+    Wo = ot.decode_rows(s, 0, ost, bits)
+    Wg = torch.empty((R, Cc), dtype=torch.float32, device="cuda")
+    L.decode_weights(Wg)
+    assert np.array_equal(Wg.cpu().numpy(), Wo)
+    xb = W.to_bf16_bits(rng.normal(0, 1, (3, Cc)).astype(np.float32))
+    y64 = O.gemv_f64(Wo, xb)
+    yabs = np.abs(Wo.astype(np.float64)) @ np.abs(W.bf16_bits_to_f32(xb).astype(np.float64)).T
+    Y = torch.empty((3, R), dtype=torch.float32, device="cuda")
+    L.gemv(x_dev(xb[:1]), Y[0])
+    check_y(Y[0].cpu().numpy(), y64[0], yabs[:, 0])
+    L.gemm_small_batch(x_dev(xb), 3, Y)
+    for b in range(3):  # every output row written once, in its own place
+        check_y(Y[b].cpu().numpy(), y64[b], yabs[:, b])
+    torch.cuda.synchronize()
+    assert L.device_error() == 0
+    L.release()
+
+
 def test_seed_zero_and_seed_fault():
     """Reading R12: a zero seed decodes as the all-zero sequence on both sides.
     Sec. 4.3: flipping one seed bit changes at most the 8 weights of its block."""
