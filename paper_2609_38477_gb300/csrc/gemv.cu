@@ -75,7 +75,7 @@ struct MultiArgs {
   int nt;
   int n;
   int ctas;
-  uint32_t zero;  // 0 at run time; keeps per-rung constants in registers
+  uint32_t zero;  // 0 at run time; keeps per-rung constants out of immediates
   int64_t cta_begin[kMaxCtas + 1];
   const TensorArgs *tens;  // layer set: nt descriptors (else t)
   const int64_t *cbd;      // layer set: ctas + 1 range starts (else cta_begin)
@@ -152,11 +152,10 @@ __device__ __forceinline__ void block_fma(const uint32_t (&w)[3], uint32_t sh, c
 }
 
 template <int K, int NB>
-__device__ __forceinline__ void run_cols(int S, const uint32_t *rowbuf, uint32_t &pos, int n,
-                                         const uint64_t *tab, const float *xc,
-                                         uint32_t z, float (&acc)[NB]) {
-  const uint32_t L = (uint32_t)(S + 4 * K + 4);
-  const RungDn<K> rc(S, z);
+__device__ __forceinline__ void run_cols(const uint4 *rent, const uint32_t *rowbuf, uint32_t &pos, int n,
+                                         const uint64_t *tab, const float *xc, float (&acc)[NB]) {
+  const RungDn<K> rc(rent);
+  const uint32_t L = rc.S + (uint32_t)(4 * K + 4);
   uint32_t w[3];
   {
     const uint32_t *q = rowbuf + (pos >> 5);
@@ -168,7 +167,10 @@ __device__ __forceinline__ void run_cols(int S, const uint32_t *rowbuf, uint32_t
     const uint32_t cur[3] = {w[0], w[1], w[2]};
     const uint32_t sh = pos;
     pos += L;
-    if (i + 1 < n) {
+    {
+      // Also after the last block: the words past a stage's end stay inside
+      // the lane's RW-word row buffer (at most (127 + ST * 44) / 32 + 3 words),
+      // and what they hold is not used.
       const uint32_t *q = rowbuf + (pos >> 5);
       w[0] = q[0];
       w[1] = q[1];
@@ -179,24 +181,39 @@ __device__ __forceinline__ void run_cols(int S, const uint32_t *rowbuf, uint32_t
 }
 
 template <int NB>
-__device__ __forceinline__ void dispatch_cols(int code, const uint32_t *rowbuf, uint32_t &pos, int n,
-                                              const uint64_t *tab, const float *xc,
-                                              uint32_t z, float (&acc)[NB]) {
-  const int S = rung_S(code);
+__device__ __forceinline__ void dispatch_cols(int code, const uint4 *rent, const uint32_t *rowbuf,
+                                              uint32_t &pos, int n, const uint64_t *tab, const float *xc,
+                                              float (&acc)[NB]) {
   switch (rung_K(code)) {
-    case 2: run_cols<2, NB>(S, rowbuf, pos, n, tab, xc, z, acc); break;
-    case 3: run_cols<3, NB>(S, rowbuf, pos, n, tab, xc, z, acc); break;
-    case 4: run_cols<4, NB>(S, rowbuf, pos, n, tab, xc, z, acc); break;
-    case 5: run_cols<5, NB>(S, rowbuf, pos, n, tab, xc, z, acc); break;
-    default: run_cols<6, NB>(S, rowbuf, pos, n, tab, xc, z, acc); break;
+    case 2: run_cols<2, NB>(rent, rowbuf, pos, n, tab, xc, acc); break;
+    case 3: run_cols<3, NB>(rent, rowbuf, pos, n, tab, xc, acc); break;
+    case 4: run_cols<4, NB>(rent, rowbuf, pos, n, tab, xc, acc); break;
+    case 5: run_cols<5, NB>(rent, rowbuf, pos, n, tab, xc, acc); break;
+    default: run_cols<6, NB>(rent, rowbuf, pos, n, tab, xc, acc); break;
+  }
+}
+
+// The per-rung constants of RungDn for every rung of a tensor (thread j < J
+// writes rung j's entry).
+__device__ __forceinline__ void store_rung_entries(const LayerArgs &p, uint32_t z, uint4 *rdn) {
+  const int j = threadIdx.x;
+  if (j >= p.J) return;
+  const int code = p.code[j], S = rung_S(code);
+  uint4 *e = rdn + j * RungDn<2>::kEntry;
+  switch (rung_K(code)) {
+    case 2: RungDn<2>(S, z).store(e); break;
+    case 3: RungDn<3>(S, z).store(e); break;
+    case 4: RungDn<4>(S, z).store(e); break;
+    case 5: RungDn<5>(S, z).store(e); break;
+    default: RungDn<6>(S, z).store(e); break;
   }
 }
 
 // Bits of the lane's row before blocks cs and ce.  Rung j spans blocks
 // [bk[j-1], bk[j]) and the breakpoints rise along the row, so the bits before
 // block x are L[0] x plus, for every breakpoint below x, the rate step dL[j]
-// times the blocks past it.  bw: the row's breakpoints as int16 pairs (zero
-// past J - 1, where dL is zero).
+// times the blocks past it.  bw: the row's breakpoints as int16 pairs (0x7fff,
+// above every block index, past J - 1, where dL is zero).
 __device__ __forceinline__ void lane_bits_before(const uint32_t (&bw)[4], const LayerArgs &p, int cs,
                                                  int ce, uint32_t &s_cs, uint32_t &s_ce) {
   s_cs = (uint32_t)p.L[0] * (uint32_t)cs;
@@ -220,7 +237,7 @@ struct Piece {
 // buffer slot carries the row data of the stage staged into it.  A warp's sums
 // go to comb[piece][warp][lane] whenever its next stage is in another piece.
 template <int NB>
-__device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t z,
+__device__ __forceinline__ void warp_round(const TensorArgs &T, int n, const uint4 *rdn,
                                            const uint64_t *tabs, uint32_t *sbuf, float *xbuf,
                                            const uint4 *rrec, const Piece *pcs, const int *pst, int np,
                                            int nst_total,
@@ -253,11 +270,9 @@ __device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t 
     int jr0 = 0, nx0 = nb;
 #pragma unroll
     for (int j = 0; j < kMaxJ - 1; ++j) {
-      const int b = (int)((bw[j >> 1] >> (16 * (j & 1))) & 0xffffu);
-      if (j < J - 1) {
-        jr0 += (b <= cs) ? 1 : 0;
-        if (b > cs) nx0 = min(nx0, b);
-      }
+      const int b = (int)((bw[j >> 1] >> (16 * (j & 1))) & 0xffffu);  // 0x7fff past J - 1
+      jr0 += (b <= cs) ? 1 : 0;
+      if (b > cs) nx0 = min(nx0, b);
     }
     const uint64_t bit_cs = roff + s_cs;
     const uint64_t b_lo = (bit_cs >> 3) & ~(uint64_t)15;
@@ -362,8 +377,8 @@ __device__ __forceinline__ void warp_round(const TensorArgs &T, int n, uint32_t 
         xo = cnt > 0 ? ra - cs : 0;
         if (!__any_sync(0xffffffffu, cnt > 0)) continue;
       }
-      dispatch_cols<NB>(p.code[j], rowbuf, pos, cnt, tabs + p.slot[j] * 512, xs + xo * 8 * NB,
-                        z, acc);
+      dispatch_cols<NB>(p.code[j], rdn + j * RungDn<2>::kEntry, rowbuf, pos, cnt,
+                        tabs + p.slot[j] * 512, xs + xo * 8 * NB, acc);
     }
     __syncwarp();
   }
@@ -501,6 +516,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ Mu
                    : "=r"(crow) : "l"(ap));
     }
     for (int i = threadIdx.x; i < np * kWarps * 32 * NB; i += kThreads) comb[i] = 0.f;
+    __shared__ uint4 rdn[kMaxJ * RungDn<2>::kEntry];
+    store_rung_entries(tens[ti].p, a.zero, rdn);
     // The round's row records (32 bytes per row of each piece; rows past R
     // repeat the group's first row), read once per round.
 #pragma unroll
@@ -513,7 +530,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_gemv(const __grid_constant__ Mu
       }
     }
     __syncthreads();
-    warp_round<NB>(T, a.n, a.zero, tabs, sbuf, xbuf, rrec, pcs, pst, np, nst_total, comb, warp, lane);
+    warp_round<NB>(T, a.n, rdn, tabs, sbuf, xbuf, rrec, pcs, pst, np, nst_total, comb, warp, lane);
     if (ck < np) srow[threadIdx.x] = crow;
     __syncthreads();
     // Row sums of the round's pieces (warps added in warp order), every (piece,

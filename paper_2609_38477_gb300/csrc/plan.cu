@@ -176,7 +176,7 @@ __global__ void k_rowrec(const int32_t *__restrict__ rowperm, const uint64_t *__
     uint32_t b[kMaxJ - 1];
 #pragma unroll
     for (int j = 0; j < kMaxJ - 1; ++j)
-      b[j] = j < J - 1 ? (uint32_t)(uint16_t)brk[r * (J - 1) + j] : 0u;
+      b[j] = j < J - 1 ? (uint32_t)(uint16_t)brk[r * (J - 1) + j] : 0x7fffu;
     rec[2 * i] = make_uint4((uint32_t)off, (uint32_t)(off >> 32), b[0] | (b[1] << 16), b[2] | (b[3] << 16));
     rec[2 * i + 1] = make_uint4(b[4] | (b[5] << 16), b[6] | (b[7] << 16), row_bits, 0u);
   }

@@ -39,7 +39,7 @@ struct LayerArgs {
   const int32_t *rowperm;   // R: order in which rows are grouped 32 to a warp
   const uint4 *rowrec;      // R x 2, at row position i (row rowperm[i]): its bit
                             // offset (words 0-1), its breakpoints as int16
-                            // pairs (words 2-5, zero past J - 1) and its bit
+                            // pairs (words 2-5, 0x7fff past J - 1) and its bit
                             // count (word 6)
   float *xperm;             // C x n: activations in permuted order, weight-major
   int32_t *counters;        // row groups: arrivals of partial sums (0 between calls)
@@ -403,6 +403,34 @@ struct RungDn {
       // Subnormal: S + j - 1 + Ko <= 22.
       const uint32_t ce = 0x80000000u | (1u << (S_ + j - 1)), co = 0x80000000u | (1u << (S_ + j - 1 + Ko));
       cinit2[j] = ((uint64_t)(co ^ z) << 32) | (uint64_t)(ce ^ z);
+    }
+  }
+  // The same constants as a table entry of 1 + 2K 16-byte words (store), read
+  // back by the second constructor.
+  static constexpr int kEntry = 1 + 2 * 6;
+  __device__ __forceinline__ void store(uint4 *e) const {
+    e[0] = make_uint4(S, e_msk, e_x, sc);
+#pragma unroll
+    for (int j = 0; j < K; ++j) {
+      e[1 + 2 * j] = make_uint4(t_msk[j], t_x[j], m_e[j], kPair ? m_o[kPair ? j : 0] : 0u);
+      e[2 + 2 * j] = make_uint4((uint32_t)cinit2[j], (uint32_t)(cinit2[j] >> 32), 0u, 0u);
+    }
+  }
+  __device__ __forceinline__ explicit RungDn(const uint4 *e) {
+    const uint4 h = e[0];
+    S = h.x;
+    e_msk = h.y;
+    e_x = h.z;
+    sc = h.w;
+#pragma unroll
+    for (int j = 0; j < K; ++j) {
+      const uint4 a = e[1 + 2 * j];
+      const uint2 b = *reinterpret_cast<const uint2 *>(e + 2 + 2 * j);
+      t_msk[j] = a.x;
+      t_x[j] = a.y;
+      m_e[j] = a.z;
+      if constexpr (kPair) m_o[j] = a.w;
+      cinit2[j] = ((uint64_t)b.y << 32) | (uint64_t)b.x;
     }
   }
 };
