@@ -251,12 +251,10 @@ __device__ __forceinline__ void warp_round(const TensorArgs &T, int n, const uin
   int jr_of[2] = {0, 0}, nxt_of[2] = {0, 0};
   uint32_t pos0[2] = {0, 0};
 
+  int pi_cur = 0;  // piece of the last stage issued (a warp's stages rise)
   auto issue = [&](int t, int sb) {
-    // Piece of stage t: the number of pieces after the first whose first
-    // stage is at or before t (independent loads, no dependent chain).
-    int pi = 0;
-#pragma unroll
-    for (int k = 1; k < CF::RG; ++k) pi += (k < np && t >= pst[k]) ? 1 : 0;
+    while (pi_cur + 1 < np && t >= pst[pi_cur + 1]) ++pi_cur;
+    const int pi = pi_cur;
     const int cs = pcs[pi].ca + (t - pst[pi]) * CF::ST, ce = min(pcs[pi].cb, cs + CF::ST);
     // The lane's row record (bit offset, breakpoints), staged for the round.
     const uint4 m0 = rrec[(pi * 32 + lane) * 2], m1 = rrec[(pi * 32 + lane) * 2 + 1];
